@@ -1,0 +1,214 @@
+"""fp64 CPU oracle for the ESTP feature path -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s cpu_baseline /
+reference arm may import this package.  It wraps ``liboracle.so`` (plain C in
+``estp_oracle.c``), which shares no code with the CUDA library.
+
+Functions and the paper passages they follow (arXiv 2608.15592):
+  token_entropy   Eq. 2-1 (Sec. 3.2)
+  attn_lse        the row normaliser of the causal softmax A (Sec. 3.1)
+  attn_colsum     sum_i A_ij of Eq. 2-0 for one layer, summed over query heads
+  importance      Eq. 2-0: S_j = C_j / (N * layers * heads)
+  pool            Eqs. 2-2, 2-3, 2-4
+  length_head     Eq. 3-2 with a linear projection
+
+bf16 arrays are passed as numpy uint16 holding the raw bfloat16 bits.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SO = os.path.join(_HERE, "_build", "liboracle.so")
+F32, BF16 = 0, 1
+
+
+def build(force: bool = False) -> str:
+    """Compile estp_oracle.c with gcc (IEEE, no FMA contraction) into _build/."""
+    src = os.path.join(_HERE, "estp_oracle.c")
+    hdr = os.path.join(_HERE, "estp_oracle.h")
+    if (not force and os.path.exists(_SO)
+            and os.path.getmtime(_SO) >= max(os.path.getmtime(src), os.path.getmtime(hdr))):
+        return _SO
+    os.makedirs(os.path.dirname(_SO), exist_ok=True)
+    tmp = _SO + f".tmp{os.getpid()}"
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+                           "-D_DEFAULT_SOURCE", "-o", tmp, src, "-lm", "-lpthread"])
+    os.replace(tmp, _SO)
+    return _SO
+
+
+class _Lib:
+    """ctypes view of one build of the oracle library."""
+
+    def __init__(self, path: str):
+        lib = ctypes.CDLL(path)
+        P, I, I64, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
+        sig = {
+            "oracle_token_entropy": [P, I, I64, I64, I64, P, I],
+            "oracle_attn_lse": [P, P, I, I, I, I, D, P, I, P, I],
+            "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
+            "oracle_importance": [P, P, I, I, I, P],
+            "oracle_pool": [P, I, I64, I64, P, P, P, I, D, D, D, P, P],
+            "oracle_length_head": [P, I, I64, P, P, P, I, P, P],
+        }
+        for name, args in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_int
+            setattr(self, name, fn)
+
+
+_lib = None
+_override = None
+
+
+def _load():
+    global _lib
+    if _override is not None:
+        return _override
+    if _lib is None:
+        _lib = _Lib(build())
+    return _lib
+
+
+class use_library:
+    """Context manager: route the functions of this module through another build
+    of the oracle (used by the tests that plant mistakes in a copy of the source)."""
+
+    def __init__(self, path: str):
+        self.lib = _Lib(path)
+
+    def __enter__(self):
+        global _override
+        self._prev, _override = _override, self.lib
+        return self
+
+    def __exit__(self, *exc):
+        global _override
+        _override = self._prev
+        return False
+
+
+def compile_source(src_text: str, out_path: str) -> str:
+    """Compile a (possibly modified) copy of estp_oracle.c with the oracle's flags."""
+    d = os.path.dirname(out_path)
+    os.makedirs(d, exist_ok=True)
+    src = os.path.join(d, "estp_oracle_variant.c")
+    with open(src, "w") as f:
+        f.write(src_text)
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+                           "-D_DEFAULT_SOURCE", "-I", _HERE, "-o", out_path, src, "-lm",
+                           "-lpthread"])
+    return out_path
+
+
+def source_text() -> str:
+    with open(os.path.join(_HERE, "estp_oracle.c")) as f:
+        return f.read()
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _dtype_code(a: np.ndarray) -> int:
+    if a.dtype == np.float32:
+        return F32
+    if a.dtype == np.uint16:
+        return BF16
+    raise TypeError(f"oracle inputs are float32 or uint16 (bf16 bits), got {a.dtype}")
+
+
+def _check(rc, name):
+    if rc != 0:
+        raise ValueError(f"{name}: invalid argument")
+
+
+def _cu(cu):
+    return np.ascontiguousarray(cu, dtype=np.int32)
+
+
+def token_entropy(logits: np.ndarray, V: int | None = None, n_threads: int = 0) -> np.ndarray:
+    """Eq. 2-1 per row of a 2-D [rows, ld] array (first V columns are the vocabulary)."""
+    logits = np.ascontiguousarray(logits)
+    rows, ld = logits.shape
+    V = ld if V is None else V
+    out = np.zeros(rows, dtype=np.float64)
+    _check(_load().oracle_token_entropy(_ptr(logits), _dtype_code(logits), rows, V, ld,
+                                        _ptr(out), n_threads), "token_entropy")
+    return out
+
+
+def attn_lse(Q, K, cu_seqlens, scale, n_threads: int = 0) -> np.ndarray:
+    """Row log-normalisers [Hq, sumT] of the causal attention of one layer."""
+    Q, K, cu = np.ascontiguousarray(Q), np.ascontiguousarray(K), _cu(cu_seqlens)
+    sumT, Hq, d = Q.shape
+    Hkv = K.shape[1]
+    out = np.zeros((Hq, sumT), dtype=np.float64)
+    _check(_load().oracle_attn_lse(_ptr(Q), _ptr(K), _dtype_code(Q), Hq, Hkv, d, float(scale),
+                                   _ptr(cu), len(cu) - 1, _ptr(out), n_threads), "attn_lse")
+    return out
+
+
+def attn_colsum(Q, K, cu_seqlens, scale, heads=None, exclude_self=False,
+                out: np.ndarray | None = None, n_threads: int = 0) -> np.ndarray:
+    """sum_{h in heads} sum_{i>=j} A^h_ij for one layer, added into ``out`` ([sumT] f64)."""
+    Q, K, cu = np.ascontiguousarray(Q), np.ascontiguousarray(K), _cu(cu_seqlens)
+    sumT, Hq, d = Q.shape
+    Hkv = K.shape[1]
+    if out is None:
+        out = np.zeros(sumT, dtype=np.float64)
+    h = None if heads is None else np.ascontiguousarray(heads, dtype=np.int32)
+    nh = Hq if h is None else len(h)
+    _check(_load().oracle_attn_colsum(_ptr(Q), _ptr(K), _dtype_code(Q), Hq, Hkv, d,
+                                      float(scale), _ptr(h), nh, _ptr(cu), len(cu) - 1,
+                                      int(bool(exclude_self)), _ptr(out), n_threads),
+           "attn_colsum")
+    return out
+
+
+def importance(C, cu_seqlens, n_layers: int, n_heads: int) -> np.ndarray:
+    """Eq. 2-0 scaling of accumulated column sums."""
+    C, cu = np.ascontiguousarray(C, dtype=np.float64), _cu(cu_seqlens)
+    out = np.zeros_like(C)
+    _check(_load().oracle_importance(_ptr(C), _ptr(cu), len(cu) - 1, n_layers, n_heads,
+                                     _ptr(out)), "importance")
+    return out
+
+
+def pool(hidden, H, S, cu_seqlens, lambda1, lambda2, alpha, D: int | None = None,
+         return_weights: bool = False):
+    """Eqs. 2-2..2-4; returns pooled [B, D] (and the weights e_i if asked)."""
+    hidden = np.ascontiguousarray(hidden)
+    rows, ldh = hidden.shape
+    D = ldh if D is None else D
+    cu = _cu(cu_seqlens)
+    B = len(cu) - 1
+    H = np.ascontiguousarray(H, dtype=np.float64)
+    S = np.ascontiguousarray(S, dtype=np.float64)
+    pooled = np.zeros((B, D), dtype=np.float64)
+    w = np.zeros(rows, dtype=np.float64) if return_weights else None
+    _check(_load().oracle_pool(_ptr(hidden), _dtype_code(hidden), D, ldh, _ptr(H), _ptr(S),
+                               _ptr(cu), B, float(lambda1), float(lambda2), float(alpha),
+                               _ptr(w), _ptr(pooled)), "pool")
+    return (pooled, w) if return_weights else pooled
+
+
+def length_head(pooled, W, bias, centers, return_probs: bool = False):
+    """Eq. 3-2: returns y_hat [B] (and p_hat [B, K] if asked)."""
+    pooled = np.ascontiguousarray(pooled, dtype=np.float64)
+    B, D = pooled.shape
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    K = W.shape[0]
+    bias = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    centers = np.ascontiguousarray(centers, dtype=np.float32)
+    y = np.zeros(B, dtype=np.float64)
+    p = np.zeros((B, K), dtype=np.float64) if return_probs else None
+    _check(_load().oracle_length_head(_ptr(pooled), B, D, _ptr(W), _ptr(bias), _ptr(centers),
+                                      K, _ptr(p), _ptr(y)), "length_head")
+    return (y, p) if return_probs else y

@@ -1,0 +1,85 @@
+/*
+ * ESTP fp64 CPU oracle -- TEST INFRASTRUCTURE ONLY.
+ *
+ * This is the plain, slow reference against which the CUDA path is checked.
+ * Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline / reference
+ * arm may load it.  It shares no code, header, table or helper with the CUDA
+ * library under paper_2608_15592_gb300/csrc, and the product path never calls it.
+ *
+ * Every function follows the definition printed in the paper (arXiv 2608.15592,
+ * "When Entropy Is Not Enough: Reclaiming Lost Semantics in LLM Output Length
+ * Prediction"), evaluated in IEEE double precision:
+ *   oracle_token_entropy       Eq. 2-1  (Sec. 3.2)
+ *   oracle_attn_lse            log-normaliser of the softmax rows of A (Sec. 3.1)
+ *   oracle_attn_colsum         the column sums of A inside Eq. 2-0 (Sec. 3.1)
+ *   oracle_importance          Eq. 2-0 (the 1/N scaling and the head/layer mean)
+ *   oracle_pool                Eqs. 2-2, 2-3, 2-4 (Sec. 3.2)
+ *   oracle_length_head         Eq. 3-2 (Sec. 3.3), linear projection + softmax
+ *
+ * Parity status: every function is pinned by the CPU tests (closed forms,
+ * invariants, brute force against independent library routines); none is
+ * "parity unpinned".
+ *
+ * Element types of the input arrays: ORACLE_F32 (IEEE binary32) or ORACLE_BF16
+ * (raw bfloat16 bits, uint16).  Both widen to double exactly.
+ * Return value of every function: 0 on success, -1 on an invalid argument.
+ * n_threads <= 0 means "one thread per online core".
+ */
+#ifndef ESTP_ORACLE_H
+#define ESTP_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { ORACLE_F32 = 0, ORACLE_BF16 = 1 };
+
+/* Eq. 2-1: H_r = -sum_v p_rv ln p_rv with p_r = softmax(logits row r), natural log.
+ * logits: n_rows rows of V values, row stride ld elements.  H_out: [n_rows]. */
+int oracle_token_entropy(const void* logits, int dtype, int64_t n_rows, int64_t V,
+                         int64_t ld, double* H_out, int n_threads);
+
+/* Row log-normaliser of causal attention for one layer:
+ * lse_out[h * sumT + i] = ln sum_{j <= i, j in prompt(i)} exp(scale * q_i^h . k_j^{h/rep}).
+ * Q: [sumT, Hq, d], K: [sumT, Hkv, d] row-major; cu_seqlens: [B+1] prompt offsets (host).
+ * All Hq heads are computed.  lse_out: [Hq, sumT]. */
+int oracle_attn_lse(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
+                    double scale, const int32_t* cu_seqlens, int B, double* lse_out,
+                    int n_threads);
+
+/* Column sums of the causal softmax attention matrix of one layer, over a set of
+ * query heads:  C_out[j] += sum_{h in heads} sum_{i >= j, i in prompt(j)} A^h_ij,
+ * A^h_ij = softmax_j(scale * q_i^h . k_j^{h/rep}) over j <= i in the same prompt.
+ * exclude_self != 0 drops the diagonal term i == j from the column sum (the row
+ * softmax itself is unchanged).  C_out: [sumT], accumulated (caller zeroes it). */
+int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
+                       double scale, const int32_t* heads, int n_heads,
+                       const int32_t* cu_seqlens, int B, int exclude_self, double* C_out,
+                       int n_threads);
+
+/* Eq. 2-0 with the head/layer mean: S_j = C_j / (N_b * n_layers * n_heads), where
+ * N_b is the length of the prompt that holds token j.  S_out: [sumT]. */
+int oracle_importance(const double* C, const int32_t* cu_seqlens, int B, int n_layers,
+                      int n_heads, double* S_out);
+
+/* Eqs. 2-2..2-4 per prompt b:  T_i = lambda1*S_i + lambda2*H_i,
+ * e_i = exp(T_i/alpha) / sum_j exp(T_j/alpha) over the prompt's tokens,
+ * pooled_b = sum_i e_i h_i.  hidden: [sumT, D] with row stride ldh elements.
+ * A prompt with no tokens pools to the zero vector.
+ * weights_out (may be NULL): [sumT] the e_i.  pooled_out: [B, D]. */
+int oracle_pool(const void* hidden, int dtype, int64_t D, int64_t ldh, const double* H,
+                const double* S, const int32_t* cu_seqlens, int B, double lambda1,
+                double lambda2, double alpha, double* weights_out, double* pooled_out);
+
+/* Eq. 3-2 with a linear projection: z = W h + bias, p = softmax(z), y = sum_k p_k c_k.
+ * pooled: [B, D]; W: [K, D] fp32; bias, centers: [K] fp32 (bias may be NULL).
+ * probs_out (may be NULL): [B, K].  yhat_out: [B]. */
+int oracle_length_head(const double* pooled, int B, int64_t D, const float* W,
+                       const float* bias, const float* centers, int K, double* probs_out,
+                       double* yhat_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

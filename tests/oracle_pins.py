@@ -1,0 +1,323 @@
+"""Pins of the fp64 oracle to facts fixed by the mathematics, not by the oracle.
+
+Each pin is a function that raises AssertionError when the oracle (whichever build
+``oracle`` currently routes to) disagrees with a closed form, an invariant, or an
+independent library routine (scipy) on tiny inputs.  ``test_oracle_pins`` runs all
+of them on the committed oracle; ``test_oracle_mutants`` runs them on copies of the
+oracle with planted mistakes and requires that some pin fails for every mistake.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+from scipy import special, stats
+
+import oracle
+from synth import f32_to_bf16_bits
+
+RTOL = 1e-11
+
+
+def _close(a, b, rtol=RTOL, atol=1e-12, what=""):
+    a, b = np.asarray(a, dtype=np.float64), np.asarray(b, dtype=np.float64)
+    assert a.shape == b.shape, f"{what}: shape {a.shape} vs {b.shape}"
+    assert np.allclose(a, b, rtol=rtol, atol=atol), (
+        f"{what}: max abs diff {np.max(np.abs(a - b)) if a.size else 0}")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# ------------------------------------------------------------- Eq. 2-1 entropy
+
+def pin_entropy_uniform():
+    """Uniform logits give H = ln V exactly (any constant, any V)."""
+    for V in (1, 7, 64, 32000, 152064):
+        for c in (0.0, -3.5, 17.0):
+            z = np.full((2, V), c, dtype=np.float32)
+            # naive summation of V terms: relative rounding bound ~ V * 2**-53
+            _close(oracle.token_entropy(z), [math.log(V)] * 2, rtol=max(1e-12, V * 2.0**-52),
+                   what=f"uniform V={V}")
+    z = f32_to_bf16_bits(np.full((1, 128256), 2.0, dtype=np.float32))
+    _close(oracle.token_entropy(z), [math.log(128256)], rtol=128256 * 2.0**-52,
+           what="uniform bf16")
+
+
+def pin_entropy_onehot_and_ties():
+    """One dominant logit gives H = 0; k tied dominant logits give H = ln k."""
+    V = 1000
+    for k in (1, 2, 3, 10):
+        z = np.zeros((1, V), dtype=np.float32)
+        z[0, np.arange(k) * 37] = 1e4
+        _close(oracle.token_entropy(z), [math.log(k)], atol=1e-12, what=f"ties k={k}")
+
+
+def pin_entropy_two_level():
+    """a entries at x and V-a at 0: H = -a p ln p - (V-a) q ln q,
+    p = e^x / (a e^x + V - a), q = 1 / (a e^x + V - a)."""
+    for V, a, x in ((50, 3, 2.5), (32000, 17, 6.0), (1000, 999, -1.25), (64, 1, 0.5)):
+        z = np.zeros((1, V), dtype=np.float32)
+        z[0, :a] = x
+        den = a * math.exp(x) + (V - a)
+        p, q = math.exp(x) / den, 1.0 / den
+        ref = -a * p * math.log(p) - (V - a) * q * math.log(q)
+        _close(oracle.token_entropy(z), [ref], rtol=max(1e-12, V * 2.0**-52),
+               what=f"two-level V={V}")
+
+
+def pin_entropy_library_bruteforce():
+    """Small V: scipy.stats.entropy of scipy.special.softmax (natural log)."""
+    rng = _rng(1)
+    for V in (1, 2, 5, 33, 64):
+        z = (rng.standard_normal((6, V)) * rng.uniform(0.1, 6, (6, 1))).astype(np.float32)
+        ref = [stats.entropy(special.softmax(r.astype(np.float64))) for r in z]
+        _close(oracle.token_entropy(z), ref, rtol=1e-11, atol=1e-13, what=f"scipy V={V}")
+
+
+def pin_entropy_shift_perm_pad():
+    """H(z + c) = H(z); H is invariant to permuting a row; columns past V are ignored."""
+    rng = _rng(2)
+    V = 300
+    z = np.round(rng.standard_normal((4, V)) * 64).astype(np.float32) / 16  # exact grid
+    H = oracle.token_entropy(z)
+    _close(oracle.token_entropy(z + np.float32(8.0)), H, rtol=1e-12, what="shift")
+    _close(oracle.token_entropy(z[:, rng.permutation(V)]), H, rtol=1e-12, what="perm")
+    padded = np.full((4, V + 13), 1e4, dtype=np.float32)
+    padded[:, :V] = z
+    _close(oracle.token_entropy(padded, V=V), H, rtol=1e-12, what="ld padding")
+
+
+# ------------------------------------------------------- Eq. 2-0 importance
+
+def _brute_colsum(Q, K, cu, scale, heads=None, exclude_self=False):
+    """Full masked score matrix per (prompt, head); rows via scipy softmax."""
+    Qd = Q.astype(np.float64) if Q.dtype != np.uint16 else _bf(Q)
+    Kd = K.astype(np.float64) if K.dtype != np.uint16 else _bf(K)
+    sumT, Hq, d = Qd.shape
+    rep = Hq // Kd.shape[1]
+    heads = range(Hq) if heads is None else heads
+    C = np.zeros(sumT)
+    for b in range(len(cu) - 1):
+        t0, t1 = cu[b], cu[b + 1]
+        if t1 == t0:
+            continue
+        T = t1 - t0
+        for h in heads:
+            S = scale * Qd[t0:t1, h] @ Kd[t0:t1, h // rep].T
+            S[np.triu_indices(T, 1)] = -np.inf
+            A = special.softmax(S, axis=1)
+            if exclude_self:
+                A[np.diag_indices(T)] = 0.0
+            C[t0:t1] += A.sum(axis=0)
+    return C
+
+
+def _bf(a):
+    from synth import bf16_bits_to_f32
+    return bf16_bits_to_f32(a).astype(np.float64)
+
+
+def _qk(rng, cu, Hq, Hkv, d, spread=1.0, dtype=np.float32):
+    sumT = int(cu[-1])
+    Q = (rng.standard_normal((sumT, Hq, d)) * spread).astype(np.float32)
+    K = (rng.standard_normal((sumT, Hkv, d)) * spread).astype(np.float32)
+    if dtype == np.uint16:
+        return f32_to_bf16_bits(Q), f32_to_bf16_bits(K)
+    return Q, K
+
+
+def pin_importance_bruteforce():
+    """T <= 16: column sums of scipy softmax rows of the causal score matrix."""
+    rng = _rng(3)
+    for cu, Hq, Hkv, d in (([0, 16], 2, 2, 8), ([0, 5, 5, 16, 17], 4, 2, 16),
+                           ([0, 9, 12], 6, 3, 4)):
+        cu = np.asarray(cu, dtype=np.int32)
+        for dt in (np.float32, np.uint16):
+            Q, K = _qk(rng, cu, Hq, Hkv, d, spread=1.5, dtype=dt)
+            sc = 1 / math.sqrt(d)
+            _close(oracle.attn_colsum(Q, K, cu, sc), _brute_colsum(Q, K, cu, sc),
+                   rtol=1e-11, what=f"brute cu={list(cu)}")
+            hs = [Hq - 1, 0]
+            _close(oracle.attn_colsum(Q, K, cu, sc, heads=hs),
+                   _brute_colsum(Q, K, cu, sc, heads=hs), rtol=1e-11, what="brute heads")
+            _close(oracle.attn_colsum(Q, K, cu, sc, exclude_self=True),
+                   _brute_colsum(Q, K, cu, sc, exclude_self=True), rtol=1e-11,
+                   what="brute exclude_self")
+
+
+def pin_importance_row_sums():
+    """Each causal softmax row sums to 1, so sum_j C_j = T_b per head; with the 1/N
+    scaling and head/layer mean, S sums to 1 over each prompt."""
+    rng = _rng(4)
+    cu = np.asarray([0, 1, 40, 41, 140], dtype=np.int32)
+    Q, K = _qk(rng, cu, 4, 1, 32, spread=2.0)
+    sc = 0.3
+    C = oracle.attn_colsum(Q, K, cu, sc)
+    C = oracle.attn_colsum(Q * np.float32(0.5), K, cu, sc, out=C)  # a second "layer"
+    for b in range(len(cu) - 1):
+        T = cu[b + 1] - cu[b]
+        _close(C[cu[b]:cu[b + 1]].sum(), 2 * 4 * T, rtol=1e-12, what="colsum total")
+    S = oracle.importance(C, cu, n_layers=2, n_heads=4)
+    for b in range(len(cu) - 1):
+        _close(S[cu[b]:cu[b + 1]].sum(), 1.0, rtol=1e-12, what="S sums to 1")
+    _close(S[cu[0]], 1.0, rtol=1e-12, what="T=1 gives S=1")
+    _close(S[cu[2]], 1.0, rtol=1e-12, what="T=1 gives S=1")
+
+
+def pin_importance_uniform_harmonic():
+    """Q = 0 (or K = 0) makes every causal row uniform, A_ij = 1/(i+1) (0-based), so
+    S_j = (H_N - H_j) / N with harmonic numbers H_n."""
+    rng = _rng(5)
+    cu = np.asarray([0, 7, 300], dtype=np.int32)
+    Q, K = _qk(rng, cu, 2, 1, 16)
+    for QQ, KK in ((np.zeros_like(Q), K), (Q, np.zeros_like(K))):
+        C = oracle.attn_colsum(QQ, KK, cu, 0.25)
+        S = oracle.importance(C, cu, n_layers=1, n_heads=2)
+        for b in range(2):
+            N = cu[b + 1] - cu[b]
+            Hn = np.concatenate([[0.0], np.cumsum(1.0 / np.arange(1, N + 1))])
+            ref = (Hn[N] - Hn[np.arange(N)]) / N
+            _close(S[cu[b]:cu[b + 1]], ref, rtol=1e-12, what="harmonic")
+
+
+def pin_importance_gqa_and_scale():
+    """GQA: query head h reads KV head h // rep -- equal to the MHA case with K heads
+    repeated; the softmax scale multiplies the scores (doubling Q == doubling scale)."""
+    rng = _rng(6)
+    cu = np.asarray([0, 12, 30], dtype=np.int32)
+    Q, K = _qk(rng, cu, 6, 2, 8)
+    Krep = np.repeat(K, 3, axis=1)
+    a = oracle.attn_colsum(Q, K, cu, 0.4)
+    _close(a, oracle.attn_colsum(Q, Krep, cu, 0.4), rtol=1e-12, what="gqa == repeated mha")
+    _close(oracle.attn_colsum(Q * np.float32(2), K, cu, 0.2), a, rtol=1e-12, what="scale")
+    for h in range(6):  # head h alone == brute force on head h with kv h//3
+        _close(oracle.attn_colsum(Q, K, cu, 0.4, heads=[h]),
+               _brute_colsum(Q, K, cu, 0.4, heads=[h]), rtol=1e-11, what=f"head {h}")
+
+
+def pin_lse_library():
+    """Row log-normalisers equal scipy.special.logsumexp over the causal prefix."""
+    rng = _rng(7)
+    cu = np.asarray([0, 3, 20], dtype=np.int32)
+    Q, K = _qk(rng, cu, 4, 2, 8, spread=2.0)
+    sc = 0.35
+    lse = oracle.attn_lse(Q, K, cu, sc)
+    Qd, Kd = Q.astype(np.float64), K.astype(np.float64)
+    for b in range(2):
+        for h in range(4):
+            for i in range(cu[b], cu[b + 1]):
+                s = sc * Kd[cu[b]:i + 1, h // 2] @ Qd[i, h]
+                _close(lse[h, i], special.logsumexp(s), rtol=1e-12, what="lse")
+
+
+def pin_importance_prompt_independence():
+    """Prompts are independent: the packed result equals each prompt run alone."""
+    rng = _rng(8)
+    cu = np.asarray([0, 10, 11, 40], dtype=np.int32)
+    Q, K = _qk(rng, cu, 2, 2, 8)
+    C = oracle.attn_colsum(Q, K, cu, 0.3)
+    for b in range(3):
+        sub = np.asarray([0, cu[b + 1] - cu[b]], dtype=np.int32)
+        _close(C[cu[b]:cu[b + 1]], oracle.attn_colsum(Q[cu[b]:cu[b + 1]], K[cu[b]:cu[b + 1]],
+                                                     sub, 0.3), rtol=1e-12, what="independent")
+
+
+# ---------------------------------------------------- Eqs. 2-2..2-4 pooling
+
+def _pool_inputs(rng, cu, D, dtype=np.float32):
+    sumT = int(cu[-1])
+    hid = rng.standard_normal((sumT, D)).astype(np.float32)
+    if dtype == np.uint16:
+        hid = f32_to_bf16_bits(hid)
+    H = rng.uniform(0, 10, sumT)
+    S = rng.uniform(0, 0.05, sumT)
+    return hid, H, S
+
+
+def pin_pool_mean():
+    """lambda1 = lambda2 = 0 gives uniform weights: the pooled vector is the mean."""
+    rng = _rng(9)
+    cu = np.asarray([0, 1, 50, 177], dtype=np.int32)
+    hid, H, S = _pool_inputs(rng, cu, 40)
+    P = oracle.pool(hid, H, S, cu, 0.0, 0.0, 1.0)
+    for b in range(3):
+        _close(P[b], hid[cu[b]:cu[b + 1]].astype(np.float64).mean(axis=0), rtol=1e-12,
+               what="mean pool")
+
+
+def pin_pool_library_weights():
+    """Weights are scipy.special.softmax((lambda1 S + lambda2 H) / alpha) per prompt,
+    and the pooled vector is the weighted sum of the rows."""
+    rng = _rng(10)
+    cu = np.asarray([0, 33, 34, 90], dtype=np.int32)
+    for dt in (np.float32, np.uint16):
+        hid, H, S = _pool_inputs(rng, cu, 24, dt)
+        hd = hid.astype(np.float64) if dt == np.float32 else _bf(hid)
+        for l1, l2, al in ((0.7, 0.3, 1.0), (0.0, 1.0, 0.5), (1.0, 0.0, 2.0), (3.0, -0.2, 0.1)):
+            P, w = oracle.pool(hid, H, S, cu, l1, l2, al, return_weights=True)
+            for b in range(3):
+                sl = slice(cu[b], cu[b + 1])
+                ref_w = special.softmax((l1 * S[sl] + l2 * H[sl]) / al)
+                _close(w[sl], ref_w, rtol=1e-12, what="weights")
+                _close(w[sl].sum(), 1.0, rtol=1e-12, what="weights sum to 1")
+                _close(P[b], ref_w @ hd[sl], rtol=1e-11, what="weighted sum")
+
+
+def pin_pool_limits():
+    """alpha -> 0 selects the argmax token's row; T = 1 returns that row; an empty
+    prompt pools to zero; permuting (T_i, h_i) pairs leaves the result unchanged."""
+    rng = _rng(11)
+    cu = np.asarray([0, 20, 21, 21, 60], dtype=np.int32)
+    hid, H, S = _pool_inputs(rng, cu, 16)
+    P = oracle.pool(hid, H, S, cu, 0.0, 1.0, 1e-6)
+    _close(P[0], hid[cu[0] + np.argmax(H[:20])], rtol=1e-12, what="alpha->0")
+    _close(P[1], hid[20], rtol=1e-12, what="T=1")
+    _close(P[2], np.zeros(16), what="empty prompt")
+    perm = np.concatenate([np.arange(0, 21), 21 + rng.permutation(39)])
+    P2 = oracle.pool(hid[perm], H[perm], S[perm], cu, 0.4, 0.6, 0.7)
+    _close(P2, oracle.pool(hid, H, S, cu, 0.4, 0.6, 0.7), rtol=1e-12, what="permutation")
+    padded = np.full((60, 16 + 5), 1e4, dtype=np.float32)  # row stride > D
+    padded[:, :16] = hid
+    _close(oracle.pool(padded, H, S, cu, 0.4, 0.6, 0.7, D=16),
+           oracle.pool(hid, H, S, cu, 0.4, 0.6, 0.7), rtol=1e-12, what="row stride")
+
+
+def pin_pool_two_token():
+    """Two tokens: e_1 = 1 / (1 + exp((T_2 - T_1)/alpha))."""
+    hid = np.asarray([[1.0, 0.0, 2.0], [0.0, 1.0, -2.0]], dtype=np.float32)
+    H = np.asarray([2.0, 5.0])
+    S = np.asarray([0.9, 0.1])
+    l1, l2, al = 2.0, 0.5, 0.8
+    T1, T2 = l1 * S[0] + l2 * H[0], l1 * S[1] + l2 * H[1]
+    e1 = 1.0 / (1.0 + math.exp((T2 - T1) / al))
+    P = oracle.pool(hid, H, S, np.asarray([0, 2], dtype=np.int32), l1, l2, al)
+    _close(P[0], e1 * hid[0].astype(np.float64) + (1 - e1) * hid[1].astype(np.float64),
+           rtol=1e-12, what="two tokens")
+
+
+# ------------------------------------------------------ Eq. 3-2 length head
+
+def pin_head():
+    """W = 0 (bias 0) gives the mean of the bin centres; a dominant logit selects its
+    centre; in general p is scipy softmax(W h + b) and y = p . c."""
+    rng = _rng(12)
+    K, D = 32, 20
+    c = ((np.arange(K) + 0.5) * 256).astype(np.float32)
+    h = rng.standard_normal((3, D))
+    y = oracle.length_head(h, np.zeros((K, D), np.float32), np.zeros(K, np.float32), c)
+    _close(y, [c.astype(np.float64).mean()] * 3, rtol=1e-12, what="W=0")
+    bias = np.zeros(K, np.float32)
+    bias[11] = 1e4
+    y = oracle.length_head(h, np.zeros((K, D), np.float32), bias, c)
+    _close(y, [float(c[11])] * 3, rtol=1e-12, what="dominant bin")
+    W = rng.standard_normal((K, D)).astype(np.float32)
+    b = rng.standard_normal(K).astype(np.float32)
+    y, p = oracle.length_head(h, W, b, c, return_probs=True)
+    ref_p = special.softmax(h @ W.astype(np.float64).T + b.astype(np.float64), axis=1)
+    _close(p, ref_p, rtol=1e-11, what="probs")
+    _close(y, ref_p @ c.astype(np.float64), rtol=1e-11, what="expectation")
+
+
+ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

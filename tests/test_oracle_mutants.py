@@ -1,0 +1,53 @@
+"""Plant plausible mistakes in copies of the oracle source and check that the pins
+catch each one (CPU only).  The committed oracle is never modified: each mutant is
+a rewritten copy compiled into a temporary directory."""
+import os
+
+import pytest
+
+import oracle
+from oracle_pins import ALL_PINS
+
+# (what the mistake is, text in estp_oracle.c, replacement)
+MUTANTS = [
+    ("entropy in bits", "H -= p * log(p);", "H -= p * log2(p);"),
+    ("entropy sign", "H -= p * log(p);", "H += p * log(p);"),
+    ("entropy unnormalised", "double p = e[v] / s;", "double p = e[v];"),
+    ("entropy ignores row stride", "int64_t off = r * c->ld;", "int64_t off = r * c->V;"),
+    ("bf16 widening shift", "[idx] << 16;", "[idx] << 15;"),
+    ("scores unscaled", "s[j] = c->scale * dot;", "s[j] = dot;"),
+    ("row sums instead of column sums", "col[j] += exp(s[j] - m) / Z;",
+     "col[i] += exp(s[j] - m) / Z;"),
+    ("softmax unnormalised", "col[j] += exp(s[j] - m) / Z;", "col[j] += exp(s[j] - m);"),
+    ("GQA head mapping", "int g = h / (c->Hq / c->Hkv);", "int g = h % c->Hkv;"),
+    ("K head ignored", "((t0 + t) * c->Hkv + g)", "((t0 + t) * c->Hkv + 0)"),
+    ("Q prompt offset dropped", "((t0 + t) * c->Hq + h)", "((t) * c->Hq + h)"),
+    ("self term never excluded", "if (c->exclude_self && j == i) continue;", ""),
+    ("lse sign", "m + log(Z);", "m - log(Z);"),
+    ("causal count divisor", "((double)N * (double)n_layers",
+     "((double)(N - j) * (double)n_layers"),
+    ("head mean dropped", "(double)n_layers * (double)n_heads)", "(double)n_layers)"),
+    ("temperature ignored", "w[i] = T / alpha;", "w[i] = T;"),
+    ("lambdas swapped", "lambda1 * S[t0 + i] + lambda2 * H[t0 + i]",
+     "lambda1 * H[t0 + i] + lambda2 * S[t0 + i]"),
+    ("pool weights unnormalised", "double e = exp(w[i] - M) / Z;", "double e = exp(w[i] - M);"),
+    ("pool ignores row stride", "(t0 + i) * ldh + x", "(t0 + i) * D + x"),
+    ("head bias dropped", "double acc = bias ? (double)bias[k] : 0.0;", "double acc = 0.0;"),
+    ("head W transposed", "W[(int64_t)k * D + x]", "W[(int64_t)x * K + k]"),
+    ("expectation over bin index", "y += p * (double)centers[k];", "y += p * (double)k;"),
+]
+
+
+@pytest.mark.parametrize("what,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(what, old, new, tmp_path):
+    src = oracle.source_text()
+    assert src.count(old) == 1, f"mutation site for '{what}' must occur exactly once"
+    so = oracle.compile_source(src.replace(old, new), str(tmp_path / "liboracle_mut.so"))
+    failed = []
+    with oracle.use_library(so):
+        for pin in ALL_PINS:
+            try:
+                pin()
+            except AssertionError:
+                failed.append(pin.__name__)
+    assert failed, f"no pin catches the planted mistake '{what}'"
