@@ -1,0 +1,171 @@
+/*
+ * estp.h -- C ABI of the ESTP feature-extraction library (GB300, sm_103a).
+ *
+ * ESTP (Entropy-and-Semantic Token Pooling, arXiv 2608.15592) turns the
+ * activations of one LLM prefill into a pooled per-prompt feature and a
+ * predicted output length:
+ *   (a) per-token next-token entropy H_i over the full vocabulary   (Eq. 2-1)
+ *   (b) per-token attention importance S_j, the attention mass key j receives
+ *       from the causal softmax rows of the selected layers/heads    (Eq. 2-0)
+ *   (c) T_i = lambda1 S_i + lambda2 H_i, e_i = softmax_i(T_i / alpha),
+ *       h = sum_i e_i h_i, and a linear length head y = sum_k p_k c_k
+ *                                                   (Eqs. 2-2..2-4, 3-2)
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Batches are varlen-packed: B prompts, prompt b owns the global token rows
+ *   cu_seqlens[b] .. cu_seqlens[b+1]-1, cu_seqlens is int32 [B+1] in DEVICE
+ *   memory with cu_seqlens[0] = 0, non-decreasing, cu_seqlens[B] = sumT.
+ *   Empty prompts (equal neighbours) are allowed.  There is no padding.
+ * - Every tensor pointer is caller-owned DEVICE memory (on the context's device)
+ *   unless a parameter says "host".  The library never frees caller memory.
+ * - All work is enqueued asynchronously on `stream` (0 = legacy default stream).
+ *   Arguments are validated on the host before any launch; a bad argument returns
+ *   ESTP_ERR_INVALID_ARG (or ESTP_ERR_UNSUPPORTED) and enqueues nothing.
+ * - Facts only the device can check (cu_seqlens contents, max_seqlen) and
+ *   bounded-wait timeouts are recorded in a device status word of the context;
+ *   estp_sync_status() synchronises the stream and returns (and clears) it.
+ *   Kernels never trap: on such an error they skip their work and return.
+ * - A context is not thread-safe; use one context per host thread / stream.
+ *   Calls on one context must be ordered (same stream, or synchronised).
+ * - Alignment: every tensor base address must be 16-byte aligned, and every row
+ *   stride (ld, ldh) times the element size a multiple of 16 bytes.
+ * - Results are deterministic: no floating-point atomics; every partial sum is
+ *   reduced in a fixed order, so repeated calls give identical bits.
+ */
+#ifndef ESTP_H
+#define ESTP_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* estp_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+    ESTP_OK = 0,
+    ESTP_ERR_INVALID_ARG = 1,  /* bad size, pointer, alignment or varlen metadata */
+    ESTP_ERR_UNSUPPORTED = 2,  /* valid request this build does not implement     */
+    ESTP_ERR_CUDA = 3,         /* a CUDA runtime call failed (message in last_error) */
+    ESTP_ERR_TIMEOUT = 4,      /* a device-side bounded wait gave up               */
+    ESTP_ERR_WORKSPACE = 5     /* workspace could not be (re)allocated             */
+} estp_status;
+
+typedef enum { ESTP_F32 = 0, ESTP_BF16 = 1 } estp_dtype;
+
+typedef struct estp_ctx estp_ctx;
+
+/* Creates a context on CUDA device `device`: a device status word and an empty,
+ * growable workspace.  *ctx receives the handle (NULL on failure). */
+estp_status estp_create(estp_ctx** ctx, int device);
+
+/* Frees the context's device memory.  Synchronises the device first.  NULL is a no-op. */
+void estp_destroy(estp_ctx* ctx);
+
+/* Human-readable message for the last non-OK status returned on this host thread
+ * (ctx may be NULL).  The pointer stays valid until the next call on the thread. */
+const char* estp_last_error(const estp_ctx* ctx);
+
+/* Synchronises `stream`, then returns and clears the device status word
+ * (ESTP_OK, ESTP_ERR_INVALID_ARG for bad varlen metadata, ESTP_ERR_TIMEOUT). */
+estp_status estp_sync_status(estp_ctx* ctx, estp_stream_t stream);
+
+/* ------------------------------------------------------------------ (a)
+ * Token entropy, Eq. 2-1 (Sec. 3.2):
+ *   entropy_out[r] = -sum_{v<V} p_rv ln p_rv,  p_r = softmax(logits[r, 0:V]),
+ * in nats, for every row r < n_rows.  Row r is the next-token distribution that
+ * the caller attributes to token r (aligning the prefill's shifted logits is the
+ * caller's job).  Rows are independent, so the varlen packing needs no metadata.
+ *   logits      : [n_rows, ld] row-major, dtype ESTP_BF16 or ESTP_F32; only the
+ *                 first V columns are read.  Values must be finite.
+ *   cu_seqlens  : optional (NULL allowed).  When given, the device checks that
+ *                 cu_seqlens[B] == n_rows and records ESTP_ERR_INVALID_ARG otherwise.
+ *   entropy_out : [n_rows] fp32.
+ * n_rows = 0 is a no-op.  Requires V >= 1, ld >= V. */
+estp_status estp_token_entropy(estp_ctx* ctx, const void* logits, estp_dtype dtype,
+                               int64_t n_rows, int64_t V, int64_t ld,
+                               const int32_t* cu_seqlens, int32_t B, float* entropy_out,
+                               estp_stream_t stream);
+
+/* ------------------------------------------------------------------ (b)
+ * Attention layout for one layer (Sec. 3.1): Q is [sumT, Hq, head_dim] and K is
+ * [sumT, Hkv, head_dim], row-major and contiguous, dtype ESTP_BF16 or ESTP_F32.
+ * Query head h reads KV head h / (Hq / Hkv) (grouped-query attention).  Scores
+ * are s_ij = softmax_scale * q_i . k_j for keys j <= i of the same prompt
+ * (causal), and A^h_ij = exp(s_ij - lse_i) with lse_i = ln sum_{j<=i} exp(s_ij).
+ * head_dim must be 64 or 128; Hq <= 256; max_seqlen >= every prompt length
+ * (checked on the device).
+ *
+ * Row log-normalisers: lse_out[h * sumT + i] = lse^h_i for every query head h,
+ * fp32 [Hq, sumT], natural log.  This is what a flash-attention prefill returns
+ * as its LSE, so callers that kept it can skip this call. */
+estp_status estp_attn_lse(estp_ctx* ctx, const void* Q, const void* K, estp_dtype dtype,
+                          int32_t Hq, int32_t Hkv, int32_t head_dim, float softmax_scale,
+                          const int32_t* cu_seqlens, int32_t B, int64_t sumT,
+                          int32_t max_seqlen, float* lse_out, estp_stream_t stream);
+
+/* Attention importance, Eq. 2-0 (Sec. 3.1), one layer per call:
+ *   C_j (+)= sum_{h in heads} sum_{i >= j, i in prompt(j)} A^h_ij
+ * into an fp32 [sumT] accumulator held by the context.  accumulate = 0 starts a
+ * new accumulation (this layer only); accumulate = 1 adds this layer.  Every call
+ * of one accumulation must use the same cu_seqlens, B, sumT and head count.
+ *   lse   : fp32 [Hq, sumT] from estp_attn_lse / the prefill, or NULL to have
+ *           the library compute it (into the workspace) first.
+ *   heads : HOST int32 [n_heads] query-head indices in [0, Hq), or NULL = all Hq.
+ *   flags : 0, or ESTP_IMP_EXCLUDE_SELF to drop the diagonal term A_jj from C_j
+ *           (the softmax rows keep it). */
+#define ESTP_IMP_EXCLUDE_SELF 1u
+estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
+                                 estp_dtype dtype, const float* lse, int32_t Hq, int32_t Hkv,
+                                 int32_t head_dim, float softmax_scale, const int32_t* heads,
+                                 int32_t n_heads, const int32_t* cu_seqlens, int32_t B,
+                                 int64_t sumT, int32_t max_seqlen, int accumulate,
+                                 uint32_t flags, estp_stream_t stream);
+
+/* Ends an accumulation: importance_out[j] = C_j / (N_b * n_layers * n_heads), N_b
+ * the length of the prompt holding token j (Eq. 2-0's 1/N, then the mean over the
+ * selected layers and heads).  n_layers = number of estp_attn_importance calls the
+ * caller means to average over (normally the calls since accumulate = 0).
+ *   importance_out : fp32 [sumT]. */
+estp_status estp_attn_importance_finalize(estp_ctx* ctx, int32_t n_layers,
+                                          float* importance_out, estp_stream_t stream);
+
+/* ------------------------------------------------------------------ (c)
+ * Mixing and pooling, Eqs. 2-2..2-4 (Sec. 3.2), then the length head, Eq. 3-2
+ * (Sec. 3.3):
+ *   T_i = lambda1 * S_i + lambda2 * H_i
+ *   e_i = exp(T_i / alpha) / sum_{j in prompt} exp(T_j / alpha)
+ *   pooled_b = sum_{i in prompt b} e_i h_i            (zero for an empty prompt)
+ *   z = W pooled_b + bias,  p = softmax(z),  y_b = sum_k p_k centers_k
+ * alpha > 0 is the temperature of Sec. 3.2 (alpha = 1 is the printed Eq. 2-3). */
+typedef struct {
+    float lambda1;  /* weight of the attention importance S (Eq. 2-2) */
+    float lambda2;  /* weight of the entropy H (Eq. 2-2)              */
+    float alpha;    /* softmax temperature (Sec. 3.2), > 0            */
+} estp_mix_params;
+
+typedef struct {
+    const float* W;        /* device fp32 [K, D] row-major                */
+    const float* bias;     /* device fp32 [K], or NULL for zero bias      */
+    const float* centers;  /* device fp32 [K] bin centres c_k (Eq. 3-2)   */
+    int32_t K;             /* number of length bins, 1..1024              */
+} estp_head;
+
+/*   hidden       : [sumT, ldh] row-major, dtype ESTP_BF16 or ESTP_F32, first D
+ *                  columns used (the prefill's hidden states h_i)
+ *   entropy      : fp32 [sumT] (H_i), importance : fp32 [sumT] (S_i)
+ *   head         : HOST pointer to the head description, or NULL for pooling only
+ *   pooled_out   : fp32 [B, D]
+ *   pred_len_out : fp32 [B] predicted lengths y_b, or NULL (requires head != NULL) */
+estp_status estp_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int64_t D,
+                      int64_t ldh, const float* entropy, const float* importance,
+                      const int32_t* cu_seqlens, int32_t B, int64_t sumT,
+                      estp_mix_params mix, const estp_head* head, float* pooled_out,
+                      float* pred_len_out, estp_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ESTP_H */

@@ -1,0 +1,250 @@
+// K-ENT: per-token entropy over the full vocabulary (Eq. 2-1, Sec. 3.2).
+//
+// For a row z of V logits, with y = z * log2(e), m = max y,
+//   s = sum_v 2^(y_v - m),  t = sum_v 2^(y_v - m) (y_v - m)
+// the entropy in nats is H = ln2 * (log2 s - t / s): p_v = 2^(y_v - m) / s and
+// -sum p ln p = ln s - (ln2 / s) sum 2^(y_v - m)(y_v - m).  All three terms are
+// built in one streaming pass, rescaling (s, t) whenever the running max grows:
+//   m' > m:  f = 2^(m - m'),  t <- f (t + (m - m') s),  s <- f s.
+//
+// Work split: the logits are n_rows x nvec 16-byte units.  The flat unit range is
+// cut into W equal pieces, one per warp, so every warp streams the same number of
+// bytes whatever V and n_rows are.  A warp finishes the rows it covers whole; a row
+// cut between warps leaves (m, s, t) partials that a second kernel merges in warp
+// order (deterministic).
+#include "estp_internal.cuh"
+
+namespace estp {
+namespace {
+
+constexpr int kEntThreads = 256;
+constexpr int kEntUnroll = 4;           // 16-byte loads in flight per lane
+constexpr float kMaskedLogit = -1e30f;  // finite: 2^(masked - m) = 0 and 0 * d = 0
+
+struct EntPart {
+    float m, s, t, pad;
+};
+
+struct EntArgs {
+    const char* base;
+    int64_t ld_bytes;
+    int64_t nvec;       // 16-byte units per row
+    int64_t V;
+    int64_t units;      // n_rows * nvec
+    int64_t n_warps;
+    float* H;
+    EntPart* part;      // [n_warps][2]: slot 0 = first segment, slot 1 = last segment
+};
+
+__device__ __forceinline__ int64_t warp_start(int64_t units, int64_t W, int64_t w) {
+    return (units * w) / W;
+}
+
+// Largest warp whose range starts at or before unit u.
+__device__ __forceinline__ int64_t unit_owner(int64_t units, int64_t W, int64_t u) {
+    int64_t w = ((u + 1) * W - 1) / units;
+    return w < W - 1 ? w : W - 1;
+}
+
+// Online update with the batch max already folded into m.
+__device__ __forceinline__ void rescale(float& m, float2& s, float2& t, float new_m) {
+    float dm = m - new_m;  // <= 0
+    float f = ex2(dm);
+    t.x = f * fmaf(dm, s.x, t.x);
+    t.y = f * fmaf(dm, s.y, t.y);
+    s.x *= f;
+    s.y *= f;
+    m = new_m;
+}
+
+__device__ __forceinline__ void accum_pair(float2 x, float m, float2& s, float2& t) {
+    const float2 l2e = make_float2(kLog2e, kLog2e);
+    const float2 nm = make_float2(-m, -m);
+    float2 d = __ffma2_rn(x, l2e, nm);  // y - m
+    float2 e = make_float2(ex2(d.x), ex2(d.y));
+    s = __fadd2_rn(s, e);
+    t = __ffma2_rn(e, d, t);
+}
+
+__device__ __forceinline__ void merge(float& m, float& s, float& t, float m2, float s2, float t2) {
+    float mm = fmaxf(m, m2);
+    float da = m - mm, db = m2 - mm;
+    float fa = ex2(da), fb = ex2(db);
+    t = fa * fmaf(da, s, t) + fb * fmaf(db, s2, t2);
+    s = fa * s + fb * s2;
+    m = mm;
+}
+
+__device__ __forceinline__ float entropy_of(float s, float t) {
+    return kLn2 * (lg2(s) - __fdividef(t, s));
+}
+
+// Masks the elements at or past V in the row's last unit (bf16: 8 per unit).
+__device__ __forceinline__ void mask_bf16(uint4& v, int valid) {
+    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+    const uint32_t neg = 0xF149u;  // bf16 bits of about -1e30
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+        if (e >= valid) {
+            uint32_t& word = w[e >> 1];
+            word = (e & 1) ? ((word & 0x0000FFFFu) | (neg << 16)) : ((word & 0xFFFF0000u) | neg);
+        }
+}
+
+__device__ __forceinline__ void mask_f32(uint4& v, int valid) {
+    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+        if (e >= valid) w[e] = __float_as_uint(kMaskedLogit);
+}
+
+// One lane's share of units [c0, c1) of one row: lane handles c0 + lane + 32k.
+template <bool kBf16>
+__device__ __forceinline__ void segment(const char* row, int64_t c0, int64_t c1, int64_t nvec,
+                                        int tail_valid, float& m, float2& s, float2& t) {
+    const int lane = threadIdx.x & 31;
+    constexpr int kPerUnit = kBf16 ? 8 : 4;
+    for (int64_t c = c0 + lane; c < c1; c += 32 * kEntUnroll) {
+        uint4 v[kEntUnroll];
+#pragma unroll
+        for (int k = 0; k < kEntUnroll; ++k) {
+            int64_t ck = c + 32 * k;
+            if (ck < c1) {
+                v[k] = ld_stream(row + ck * 16);
+                if (ck == nvec - 1 && tail_valid < kPerUnit) {
+                    if (kBf16) mask_bf16(v[k], tail_valid); else mask_f32(v[k], tail_valid);
+                }
+            } else {
+                if (kBf16) v[k] = make_uint4(0xF149F149u, 0xF149F149u, 0xF149F149u, 0xF149F149u);
+                else {
+                    uint32_t n = __float_as_uint(kMaskedLogit);
+                    v[k] = make_uint4(n, n, n, n);
+                }
+            }
+        }
+        // batch max (one rescale per batch of kEntUnroll units)
+        float bm;
+        if (kBf16) {
+            __nv_bfloat162 mx = *reinterpret_cast<__nv_bfloat162*>(&v[0].x);
+#pragma unroll
+            for (int k = 0; k < kEntUnroll; ++k) {
+                const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v[k]);
+#pragma unroll
+                for (int q = (k == 0 ? 1 : 0); q < 4; ++q) mx = __hmax2(mx, p[q]);
+            }
+            bm = fmaxf(__low2float(mx), __high2float(mx));
+        } else {
+            bm = __uint_as_float(v[0].x);
+#pragma unroll
+            for (int k = 0; k < kEntUnroll; ++k) {
+                bm = fmaxf(bm, __uint_as_float(v[k].x));
+                bm = fmaxf(bm, __uint_as_float(v[k].y));
+                bm = fmaxf(bm, __uint_as_float(v[k].z));
+                bm = fmaxf(bm, __uint_as_float(v[k].w));
+            }
+        }
+        float new_m = fmaxf(m, bm * kLog2e);
+        rescale(m, s, t, new_m);
+#pragma unroll
+        for (int k = 0; k < kEntUnroll; ++k) {
+            if (kBf16) {
+                accum_pair(make_float2(bf16lo(v[k].x), bf16hi(v[k].x)), m, s, t);
+                accum_pair(make_float2(bf16lo(v[k].y), bf16hi(v[k].y)), m, s, t);
+                accum_pair(make_float2(bf16lo(v[k].z), bf16hi(v[k].z)), m, s, t);
+                accum_pair(make_float2(bf16lo(v[k].w), bf16hi(v[k].w)), m, s, t);
+            } else {
+                accum_pair(make_float2(__uint_as_float(v[k].x), __uint_as_float(v[k].y)), m, s, t);
+                accum_pair(make_float2(__uint_as_float(v[k].z), __uint_as_float(v[k].w)), m, s, t);
+            }
+        }
+    }
+}
+
+template <bool kBf16>
+__global__ void __launch_bounds__(kEntThreads) entropy_kernel(EntArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w = (int64_t)blockIdx.x * (kEntThreads / 32) + (threadIdx.x >> 5);
+    if (w >= a.n_warps) return;
+    constexpr int kPerUnit = kBf16 ? 8 : 4;
+    const int tail_valid = (int)(a.V - (a.nvec - 1) * kPerUnit);
+    const int64_t start = warp_start(a.units, a.n_warps, w);
+    const int64_t end = warp_start(a.units, a.n_warps, w + 1);
+    int64_t u = start;
+    while (u < end) {
+        const int64_t r = u / a.nvec;
+        const int64_t row_u0 = r * a.nvec;
+        const int64_t seg_end = min(end, row_u0 + a.nvec);
+        const int64_t c0 = u - row_u0, c1 = seg_end - row_u0;
+        float m = kMaskedLogit;
+        float2 s = make_float2(0.f, 0.f), t = make_float2(0.f, 0.f);
+        segment<kBf16>(a.base + r * a.ld_bytes, c0, c1, a.nvec, tail_valid, m, s, t);
+        float ss = s.x + s.y, tt = t.x + t.y;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+            float s2 = __shfl_xor_sync(0xffffffffu, ss, off);
+            float t2 = __shfl_xor_sync(0xffffffffu, tt, off);
+            merge(m, ss, tt, m2, s2, t2);
+        }
+        if (lane == 0) {
+            if (c0 == 0 && c1 == a.nvec) {
+                a.H[r] = entropy_of(ss, tt);
+            } else {
+                a.part[w * 2 + (u == start ? 0 : 1)] = EntPart{m, ss, tt, 0.f};
+            }
+        }
+        u = seg_end;
+    }
+}
+
+// Rows cut between warps: merge the partials of the covering warps in warp order.
+__global__ void entropy_merge_kernel(EntArgs a, int64_t n_rows, const int32_t* cu, int B,
+                                     int* status) {
+    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (r == 0 && cu != nullptr && (int64_t)cu[B] != n_rows) report(status, ESTP_ERR_INVALID_ARG);
+    if (r >= n_rows) return;
+    const int64_t w_lo = unit_owner(a.units, a.n_warps, r * a.nvec);
+    const int64_t w_hi = unit_owner(a.units, a.n_warps, (r + 1) * a.nvec - 1);
+    if (w_lo == w_hi) return;  // one warp covered the whole row and wrote H[r]
+    float m = kMaskedLogit, s = 0.f, t = 0.f;
+    for (int64_t w = w_lo; w <= w_hi; ++w) {
+        const int64_t st = warp_start(a.units, a.n_warps, w);
+        if (st == warp_start(a.units, a.n_warps, w + 1)) continue;  // empty range
+        const EntPart p = a.part[w * 2 + (st / a.nvec == r ? 0 : 1)];
+        merge(m, s, t, p.m, p.s, p.t);
+    }
+    a.H[r] = entropy_of(s, t);
+}
+
+}  // namespace
+
+estp_status launch_entropy(estp_ctx* ctx, const void* logits, estp_dtype dtype, int64_t n_rows,
+                           int64_t V, int64_t ld, const int32_t* cu, int32_t B, float* H,
+                           cudaStream_t st) {
+    const int per_unit = dtype == ESTP_BF16 ? 8 : 4;
+    EntArgs a;
+    a.base = static_cast<const char*>(logits);
+    a.ld_bytes = ld * esize(dtype);
+    a.nvec = (V + per_unit - 1) / per_unit;
+    a.V = V;
+    a.units = n_rows * a.nvec;
+    int occ = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &occ, dtype == ESTP_BF16 ? entropy_kernel<true> : entropy_kernel<false>, kEntThreads, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
+    int64_t max_warps = (int64_t)ctx->num_sms * (occ > 0 ? occ : 1) * (kEntThreads / 32);
+    a.n_warps = a.units < max_warps ? a.units : max_warps;
+    estp_status s = ws_reserve(ctx, sizeof(EntPart) * 2 * (size_t)a.n_warps);
+    if (s != ESTP_OK) return s;
+    a.part = static_cast<EntPart*>(ctx->ws);
+    a.H = H;
+    const int64_t blocks = (a.n_warps + kEntThreads / 32 - 1) / (kEntThreads / 32);
+    if (dtype == ESTP_BF16) entropy_kernel<true><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
+    else entropy_kernel<false><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
+    const int64_t mblocks = (n_rows + 255) / 256;
+    entropy_merge_kernel<<<(unsigned)mblocks, 256, 0, st>>>(a, n_rows, cu, B, ctx->status);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "entropy launch");
+}
+
+}  // namespace estp

@@ -1,0 +1,174 @@
+"""Attention importance (LSE + column sums + finalize) against the oracle (GPU)."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_util import assert_importance
+from synth import device as sd
+from synth import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _wl(dtype, lens, Hq, Hkv, d, seed=21, sinks=0, layers=1):
+    w = W.Workload("imp", seed=seed, B=len(lens), T_lo=1, T_hi=1, dtype=dtype, V=8,
+                   n_layers_model=layers, layers_used=layers, Hq=Hq, Hkv=Hkv, d=d, D=8,
+                   sinks=sinks)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    return w, cu
+
+
+def _qk(w, cu, layer):
+    """Q, K on the host (numpy) and device (torch) for explicit cu_seqlens."""
+    sumT = int(cu[-1])
+    rows = np.arange(sumT)
+    key_q, key_k = w.key_q(layer), w.key_k(layer)
+    Qh = synth.round_to(synth.normal(key_q, np.arange(sumT * w.Hq * w.d)), w.dtype).reshape(sumT, w.Hq, w.d)
+    K64 = synth.normal(key_k, np.arange(sumT * w.Hkv * w.d)).reshape(sumT, w.Hkv, w.d)
+    if w.sinks:
+        for b in range(len(cu) - 1):
+            K64[cu[b]:min(cu[b] + w.sinks, cu[b + 1])] *= w.sink_scale
+    Kh = synth.round_to(K64, w.dtype).reshape(sumT, w.Hkv, w.d)
+    tdt = torch.bfloat16 if w.dtype == synth.BF16 else torch.float32
+    if w.dtype == synth.BF16:
+        Qd = torch.from_numpy(Qh.view(np.int16)).view(tdt).cuda()
+        Kd = torch.from_numpy(Kh.view(np.int16)).view(tdt).cuda()
+    else:
+        Qd, Kd = torch.from_numpy(Qh).cuda(), torch.from_numpy(Kh).cuda()
+    return Qh, Kh, Qd, Kd
+
+
+def _run(cuda_lib, w, cu, layers, heads=None, exclude_self=False, supply_lse=False):
+    ctx = cuda_lib.Context(0)
+    cu_d = torch.as_tensor(cu, device="cuda")
+    maxT = int(np.diff(cu).max())
+    sumT = int(cu[-1])
+    C = np.zeros(sumT)
+    for n, layer in enumerate(layers):
+        Qh, Kh, Qd, Kd = _qk(w, cu, layer)
+        lse = None
+        if supply_lse:
+            lse = torch.as_tensor(oracle.attn_lse(Qh, Kh, cu, 1 / math.sqrt(w.d)),
+                                  dtype=torch.float32, device="cuda").contiguous()
+        ctx.attn_importance(Qd, Kd, cu_d, maxT, lse=lse, heads=heads, accumulate=n > 0,
+                            exclude_self=exclude_self)
+        oracle.attn_colsum(Qh, Kh, cu, 1 / math.sqrt(w.d), heads=heads,
+                           exclude_self=exclude_self, out=C)
+    S = ctx.attn_importance_finalize(len(layers), sumT)
+    ctx.sync_status()
+    nh = w.Hq if heads is None else len(heads)
+    ref = oracle.importance(C, cu, len(layers), nh)
+    return S.cpu().numpy(), ref
+
+
+CASES = [
+    # lens, Hq, Hkv, d
+    ([1], 2, 1, 64),
+    ([5, 0, 130, 1], 4, 4, 64),
+    ([129, 300], 7, 1, 128),
+    ([700], 8, 1, 128),
+    ([257, 64, 63, 513], 28, 4, 128),
+    ([1100], 4, 2, 64),
+]
+
+
+@pytest.mark.parametrize("dtype", [synth.BF16, synth.F32])
+@pytest.mark.parametrize("lens,Hq,Hkv,d", CASES, ids=[f"c{i}" for i in range(len(CASES))])
+def test_importance_cases(cuda_lib, dtype, lens, Hq, Hkv, d):
+    w, cu = _wl(dtype, lens, Hq, Hkv, d)
+    S, ref = _run(cuda_lib, w, cu, [0])
+    assert_importance(S, ref)
+    for b in range(len(lens)):
+        if lens[b]:
+            assert abs(S[cu[b]:cu[b + 1]].sum() - 1.0) < 1e-4
+
+
+@pytest.mark.parametrize("dtype", [synth.BF16, synth.F32])
+def test_importance_layers_heads_self(cuda_lib, dtype):
+    w, cu = _wl(dtype, [300, 45, 200], 8, 2, 128, sinks=4, layers=3)
+    S, ref = _run(cuda_lib, w, cu, [0, 1, 2])
+    assert_importance(S, ref)
+    S, ref = _run(cuda_lib, w, cu, [1], heads=[5, 0, 7])
+    assert_importance(S, ref)
+    S, ref = _run(cuda_lib, w, cu, [2], exclude_self=True)
+    assert_importance(S, ref)
+    S, ref = _run(cuda_lib, w, cu, [0, 2], supply_lse=True)
+    assert_importance(S, ref)
+
+
+def test_lse_against_oracle(cuda_lib):
+    for dtype in (synth.BF16, synth.F32):
+        w, cu = _wl(dtype, [1, 257, 90], 6, 2, 64, sinks=2)
+        Qh, Kh, Qd, Kd = _qk(w, cu, 0)
+        ctx = cuda_lib.Context(0)
+        lse = ctx.attn_lse(Qd, Kd, torch.as_tensor(cu, device="cuda"), 257)
+        ctx.sync_status()
+        ref = oracle.attn_lse(Qh, Kh, cu, 1 / math.sqrt(64))
+        err = np.max(np.abs(lse.cpu().numpy() - ref) / (1 + np.abs(ref)))
+        assert err < 1e-5, err
+
+
+def test_importance_deterministic(cuda_lib):
+    w, cu = _wl(synth.BF16, [900, 333], 28, 4, 128)
+    _, _, Qd, Kd = _qk(w, cu, 0)
+    ctx = cuda_lib.Context(0)
+    cu_d = torch.as_tensor(cu, device="cuda")
+    outs = []
+    for _ in range(2):
+        ctx.attn_importance(Qd, Kd, cu_d, 900)
+        outs.append(ctx.attn_importance_finalize(1, int(cu[-1])))
+    ctx.sync_status()
+    assert torch.equal(outs[0], outs[1])
+
+
+def test_importance_device_checks(cuda_lib):
+    w, cu = _wl(synth.BF16, [100, 50], 4, 2, 64)
+    _, _, Qd, Kd = _qk(w, cu, 0)
+    ctx = cuda_lib.Context(0)
+    cu_d = torch.as_tensor(cu, device="cuda")
+    ctx.attn_importance(Qd, Kd, cu_d, 99)  # max_seqlen below a prompt length
+    with pytest.raises(cuda_lib.EstpError) as e:
+        ctx.sync_status()
+    assert e.value.status == cuda_lib.ESTP_ERR_INVALID_ARG
+    with pytest.raises(cuda_lib.EstpError):
+        ctx.attn_importance(Qd, Kd, cu_d, 100, heads=[4])  # head out of range
+    fresh = cuda_lib.Context(0)
+    with pytest.raises(cuda_lib.EstpError):
+        fresh.attn_importance(Qd, Kd, cu_d, 100, accumulate=True)  # no open accumulation
+    fresh.attn_importance(Qd, Kd, cu_d, 100)
+    with pytest.raises(cuda_lib.EstpError):  # a different prompt set cannot join it
+        fresh.attn_importance(Qd[:100], Kd[:100], cu_d[:2], 100, accumulate=True)
+
+
+@pytest.mark.parametrize("w", [W.C1, W.C2], ids=lambda w: w.name)
+def test_importance_workload(cuda_lib, w):
+    """Whole workload, all selected layers and heads on the GPU (the bench's launch
+    configuration).  Oracle on every prompt for the small case; for the full-size one on
+    the shortest and longest prompts; S sums to 1 over every prompt."""
+    cu = w.cu_seqlens()
+    sumT = int(cu[-1])
+    maxT = int(np.diff(cu).max())
+    ctx = cuda_lib.Context(0)
+    cu_d = sd.cu_seqlens(w)
+    for n, layer in enumerate(w.layers):
+        Q, K = sd.qk(w, layer)
+        ctx.attn_importance(Q, K, cu_d, maxT, accumulate=n > 0)
+    S = ctx.attn_importance_finalize(len(w.layers), sumT).cpu().numpy()
+    ctx.sync_status()
+    for b in range(w.B):
+        assert abs(S[cu[b]:cu[b + 1]].sum() - 1.0) < 1e-4
+    lens = np.diff(cu)
+    pick = np.arange(w.B) if w.B <= 2 else sorted({int(np.argmin(lens)), int(np.argmax(lens))})
+    for b in pick:
+        rows = np.arange(cu[b], cu[b + 1])
+        sub = np.asarray([0, len(rows)], dtype=np.int32)
+        C = np.zeros(len(rows))
+        for layer in w.layers:
+            Qh, Kh = W.host_qk(w, layer, rows)
+            oracle.attn_colsum(Qh, Kh, sub, w.scale, out=C)
+        ref = oracle.importance(C, sub, len(w.layers), w.Hq)
+        assert_importance(S[rows], ref)
