@@ -1,0 +1,469 @@
+"""Throughput of the ESTP feature path on GB300 (prompt tokens/s).
+
+One step = the whole hot path over one batch of the Qwen2.5-7B-shaped workload
+(16 varlen prompts, T ~ U[256, 2048], vocab 152064, last 4 layers, 28/4 heads,
+head_dim 128, hidden 3584, bf16):
+  token entropy over every row of the logits              (estp_token_entropy)
+  per layer: row log-normalisers + causal column sums     (estp_attn_lse, estp_attn_importance)
+  importance scaling                                      (estp_attn_importance_finalize)
+  mixing, tempered softmax, pooling and the length head   (estp_pool)
+Inputs are synthetic (seeded generator), resident in HBM before timing; together
+they are ~6.4 GB, far larger than the 129 MB L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the fp64 CPU oracle (the only other implementation of this
+path) on a bounded sample of the same workload.  Under torchrun each rank runs its
+own batch (same shape, rank-specific seed): prompts are independent, so there is no
+data-path collective and the scaling is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "prompt tokens/s through ESTP features (1 GB300)"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p.get("bf16_tflops_sustained"), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# --------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.lines, self.proc = index, [], None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ workload
+def workload_for_rank(rank: int):
+    from synth import workloads as W
+    w = W.C2
+    if rank:
+        import dataclasses
+        w = dataclasses.replace(w, seed=w.seed + 1000 * rank)
+    return w
+
+
+def algorithmic(w, cu):
+    """Per-launch algorithmic work of each kernel of one step."""
+    import numpy as np
+    lens = np.diff(cu).astype(np.float64)
+    sumT = float(lens.sum())
+    esz = 2 if w.dtype == "bf16" else 4
+    attn_flops = float(w.Hq * 2 * w.d * np.sum(lens * (lens + 1) / 2))  # one QK^T pass
+    return {
+        "entropy": {"bytes": sumT * w.V * esz + 4 * sumT},
+        "lse": {"flops": attn_flops},
+        "importance": {"flops": attn_flops},
+        "pool": {"bytes": sumT * w.D * esz + 8 * sumT + w.B * w.D * 4},
+    }
+
+
+def traffic_for(kernel: str):
+    """dram bytes per launch from a committed ncu summary, if the kernel's source has
+    not changed since the capture; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            t = json.load(f)[kernel]
+        src = os.path.join(ROOT, "paper_2608_15592_gb300", "csrc", t["source"])
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        return t["dram_bytes_per_launch"] if h == t["source_sha256_16"] else None
+    except Exception:
+        return None
+
+
+class Step:
+    """Device tensors of one batch plus the calls of one step."""
+
+    def __init__(self, estp, w, device):
+        import numpy as np
+        import torch
+        from synth import device as sd
+        self.estp, self.w = estp, w
+        self.cu_h = w.cu_seqlens()
+        self.sumT = int(self.cu_h[-1])
+        self.maxT = int(np.diff(self.cu_h).max())
+        self.cu = sd.cu_seqlens(w, device)
+        self.logits = sd.logits(w, 0, self.sumT, device=device)
+        self.Q, self.K = [], []
+        for layer in w.layers:
+            q, k = sd.qk(w, layer, device)
+            self.Q.append(q)
+            self.K.append(k)
+        self.hidden = sd.hidden(w, device)
+        Wt, b, c = sd.head(w, device)
+        self.head = estp.Head(Wt, b, c)
+        self.H = torch.empty(self.sumT, dtype=torch.float32, device=device)
+        self.S = torch.empty(self.sumT, dtype=torch.float32, device=device)
+        self.lse = torch.empty(w.Hq, self.sumT, dtype=torch.float32, device=device)
+        self.pooled = torch.empty(w.B, w.D, dtype=torch.float32, device=device)
+        self.pred = torch.empty(w.B, dtype=torch.float32, device=device)
+        self.ctx = estp.Context(torch.cuda.current_device())
+        n_layers = len(w.layers)
+        # launches per step: entropy 2; per layer lse 2 + importance 3; finalize 1; pool 4
+        self.launches = 2 + n_layers * 5 + 1 + 4
+
+    def run(self, ev=None):
+        """One step on the current stream; ev: dict of (start, end) events per kernel."""
+        w, c = self.w, self.ctx
+
+        def mark(name, i):
+            if ev is not None:
+                ev[name][i].record()
+
+        mark("entropy", 0)
+        c.token_entropy(self.logits, cu_seqlens=self.cu, out=self.H)
+        mark("entropy", 1)
+        for n in range(len(w.layers)):
+            mark("lse", 2 * n)
+            c.attn_lse(self.Q[n], self.K[n], self.cu, self.maxT, out=self.lse)
+            mark("lse", 2 * n + 1)
+            mark("importance", 2 * n)
+            c.attn_importance(self.Q[n], self.K[n], self.cu, self.maxT, lse=self.lse,
+                              accumulate=n > 0)
+            mark("importance", 2 * n + 1)
+        c.attn_importance_finalize(len(w.layers), self.sumT, out=self.S)
+        mark("pool", 0)
+        c.pool(self.hidden, self.H, self.S, self.cu, w.lambda1, w.lambda2, w.alpha,
+               head=self.head, pooled=self.pooled, pred=self.pred)
+        mark("pool", 1)
+
+
+# ------------------------------------------------------------------ our arm
+def run_ours(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import paper_2608_15592_gb300 as estp
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = workload_for_rank(rank)
+    st = Step(estp, w, dev)
+    torch.cuda.synchronize()
+    n_layers = len(w.layers)
+    per_step_launch_counts = {"entropy": 1, "lse": n_layers, "importance": n_layers, "pool": 1}
+
+    def new_events(k):
+        return {name: [torch.cuda.Event(enable_timing=True) for _ in range(2 * n * k)]
+                for name, n in per_step_launch_counts.items()}
+
+    for _ in range(args.warmup):
+        st.run()
+    st.ctx.sync_status()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev_steps = [new_events(1) for _ in range(K)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        start.record()
+        for k in range(K):
+            st.run(ev_steps[k])
+        end.record()
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    st.ctx.sync_status()
+    ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+        n = torch.tensor([float(st.sumT)], device=dev)
+        torch.distributed.all_reduce(n)
+        tokens = float(n.item())
+    else:
+        tokens = float(st.sumT)
+    ms_per_step = ms / K
+    value = tokens * K / (ms / 1e3)
+
+    # per-kernel averages over the timed region
+    kern_ms = {}
+    for name, n in per_step_launch_counts.items():
+        tot = 0.0
+        for ev in ev_steps:
+            for i in range(n):
+                tot += ev[name][2 * i].elapsed_time(ev[name][2 * i + 1])
+        kern_ms[name] = tot / (K * n)
+    alg = algorithmic(w, st.cu_h)
+    hbm, bf16, bf16_sus, peak_src = _peaks()
+    kernels = {}
+    for name, ms_k in kern_ms.items():
+        a = alg[name]
+        if "bytes" in a:
+            achieved = a["bytes"] / (ms_k / 1e3) / 1e9
+            kernels[name] = {"ms": ms_k, "bound": "hbm", "achieved": achieved, "unit": "GB/s",
+                             "frac": achieved / hbm}
+        else:
+            achieved = a["flops"] / (ms_k / 1e3) / 1e12
+            kernels[name] = {"ms": ms_k, "bound": "tensor", "achieved": achieved,
+                             "unit": "TFLOP/s", "frac": achieved / bf16_sus}
+    step_share = {k: kern_ms[k] * per_step_launch_counts[k] for k in kern_ms}
+    dom = max(step_share, key=step_share.get)
+    dk = kernels[dom]
+    roofline = {"kernel": dom, "bound": dk["bound"], "achieved": dk["achieved"],
+                "peak": hbm if dk["bound"] == "hbm" else bf16_sus, "unit": dk["unit"],
+                "frac": dk["frac"], "traffic": traffic_for(dom),
+                "peak_source": f"{peak_src} ({'hbm_gbs' if dk['bound'] == 'hbm' else 'bf16_tflops_sustained'})"}
+
+    e2e = run_e2e(args, st, estp, dev, world)
+    clocks = clk.summary()
+    del st
+    if rank != 0:
+        return None
+    cpu = None if (world > 1 or args.no_cpu_baseline) else cpu_baseline(w, args.cpu_seconds)
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "sum_tokens_per_gpu": st_tokens(w),
+                   "seq_len": f"U[{w.T_lo},{w.T_hi}]", "vocab": w.V, "layers": len(w.layers),
+                   "Hq": w.Hq, "Hkv": w.Hkv, "head_dim": w.d, "hidden": w.D,
+                   "mix": [w.lambda1, w.lambda2, w.alpha], "seed": w.seed,
+                   "parallelism": f"dp{world} (independent prompts)",
+                   "l2": "inputs larger than L2 (~6.4 GB per step), no flush"},
+        "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": st_launches(w) * K, "clocks": clocks,
+    }
+
+
+def st_tokens(w):
+    return int(w.cu_seqlens()[-1])
+
+
+def st_launches(w):
+    return 2 + len(w.layers) * 5 + 1 + 4
+
+
+def run_e2e(args, st, estp, dev, world):
+    """Same metric through the public API with host buffers: every step copies the
+    inputs from pinned host memory and reads the predictions and pooled features back."""
+    import torch
+    host = {}
+    for name, t in [("logits", st.logits), ("hidden", st.hidden)] + \
+                   [(f"q{i}", q) for i, q in enumerate(st.Q)] + [(f"k{i}", k) for i, k in enumerate(st.K)]:
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        host[name] = h
+    pred_h = torch.empty(st.pred.shape, dtype=torch.float32, pin_memory=True)
+    pooled_h = torch.empty(st.pooled.shape, dtype=torch.float32, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = pred_h.numel() * 4 + pooled_h.numel() * 4
+
+    def step():
+        st.logits.copy_(host["logits"], non_blocking=True)
+        st.hidden.copy_(host["hidden"], non_blocking=True)
+        for i in range(len(st.Q)):
+            st.Q[i].copy_(host[f"q{i}"], non_blocking=True)
+            st.K[i].copy_(host[f"k{i}"], non_blocking=True)
+        st.run()
+        pred_h.copy_(st.pred, non_blocking=True)
+        pooled_h.copy_(st.pooled, non_blocking=True)
+
+    for _ in range(max(1, min(args.warmup, 2))):
+        step()
+    torch.cuda.synchronize()
+    K = max(1, min(args.steps, 5))
+    if world > 1:
+        torch.distributed.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(K):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": st.sumT * world * K / (ms / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": K}
+
+
+# ------------------------------------------------------------- CPU oracle arm
+def oracle_sample_rate(w, seconds_hint: float):
+    """Time the fp64 oracle on a bounded sample of the workload and extrapolate to
+    tokens/s by algorithmic work.  Returns (tokens/s, description, threads)."""
+    import numpy as np
+    import oracle
+    from synth import workloads as W
+    n_threads = os.cpu_count() or 1
+    cu = w.cu_seqlens()
+    lens = np.diff(cu)
+    sumT = int(cu[-1])
+    # entropy on n_rows rows
+    n_rows = max(16, int(4 * n_threads))
+    x = W.host_logits(w, np.arange(n_rows))
+    t0 = time.perf_counter()
+    H = oracle.token_entropy(x, n_threads=n_threads)
+    t_ent = (time.perf_counter() - t0) * sumT / n_rows
+    # importance on the shortest prompt, all selected layers and heads (+ its LSE cost
+    # is part of the same row softmax in the oracle)
+    b = int(np.argmin(lens))
+    rows = np.arange(cu[b], cu[b + 1])
+    sub = np.asarray([0, len(rows)], dtype=np.int32)
+    layers = w.layers[:max(1, min(len(w.layers), int(seconds_hint // 5) or 1))]
+    C = np.zeros(len(rows))
+    qk = [W.host_qk(w, layer, rows) for layer in layers]
+    t0 = time.perf_counter()
+    for Qh, Kh in qk:
+        oracle.attn_colsum(Qh, Kh, sub, w.scale, out=C, n_threads=n_threads)
+    t_imp_s = time.perf_counter() - t0
+    work = lambda L: np.sum(L * (L + 1) / 2.0)
+    t_imp = t_imp_s * (work(lens) * len(w.layers)) / (work(np.asarray([len(rows)])) * len(layers))
+    # pooling + head on the same prompt
+    hid = W.host_hidden(w, rows)
+    Wt, bb, cc = w.head_params()
+    t0 = time.perf_counter()
+    P = oracle.pool(hid, H[:1].repeat(len(rows)), C, sub, w.lambda1, w.lambda2, w.alpha)
+    oracle.length_head(P, Wt, bb, cc)
+    t_pool = (time.perf_counter() - t0) * sumT / len(rows)
+    total = t_ent + t_imp + t_pool
+    desc = (f"entropy {n_rows} rows; importance prompt of {len(rows)} tokens x {len(layers)} "
+            f"layer(s) x {w.Hq} heads; pooling+head that prompt; extrapolated by algorithmic work "
+            f"to the {sumT}-token batch (entropy {t_ent:.1f}s, importance {t_imp:.1f}s, "
+            f"pool {t_pool:.2f}s per batch)")
+    return sumT / total, desc, n_threads
+
+
+def cpu_baseline(w, seconds_hint):
+    v, desc, n = oracle_sample_rate(w, seconds_hint)
+    return {"value": v, "unit": UNIT, "cores": n, "kind": "oracle", "sample": desc}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    w = workload_for_rank(0)
+    vals = []
+    desc, n = "", 1
+    for i in range(args.warmup + args.steps):
+        v, desc, n = oracle_sample_rate(w, min(args.cpu_seconds, 5.0))
+        if i >= args.warmup:
+            vals.append(v)
+    value = statistics.mean(vals)
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": st_tokens(w) / value * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": w.name, "B": w.B,
+                                        "sum_tokens_per_gpu": st_tokens(w)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": n, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="rough CPU time budget of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+        if out is not None:
+            print(json.dumps(out), flush=True)
+        return
+    import __graft_entry__
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    import torch
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+        torch.distributed.barrier()
+        if rank != 0:
+            __graft_entry__.build()
+    out = run_ours(args, rank, world, local_rank)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
