@@ -117,6 +117,27 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
     return true;
 }
 
+// Bounded wait that ignores the abort flag (used to drain outstanding MMAs).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* status) {
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > kWaitCycles) {
+            report(status, ESTP_ERR_TIMEOUT);
+            return;
+        }
+    }
+}
+
+// Warp-uniform bounded wait: lane 0 polls, every lane gets the same answer.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          int* status) {
+    bool r = false;
+    if ((threadIdx.x & 31) == 0) r = wait_bar(bar, parity, abort_flag, status);
+    r = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0;
+    __syncwarp();
+    return r;
+}
+
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
                                             uint64_t* bar) {
     asm volatile(
@@ -366,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (issued) {  // every MMA done before the TMEM is released
                 mma_commit(drain);
-                wait_bar(drain, 0, abort_flag, a.status);
+                drain_wait(drain, 0, a.status);
             }
         }
     } else {
@@ -377,8 +398,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* nl = nl_all + (warp - kEpiWarp0) * 64;
         long long step = 0;
         int it = 0;
-        bool ok = true;
-        for (int item = blockIdx.x; item < total && ok; item += gridDim.x, ++it) {
+        bool ok = true;  // false once any wait gave up: the loops then run without waiting
+        for (int item = blockIdx.x; item < total; item += gridDim.x, ++it) {
             const TcItem t = make_item<MODE>(a, item);
             float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
             float m = -1e30f, ssum = 0.f;          // LSE mode
@@ -403,10 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (s + 1 < t.n_steps) load_nl(s + 1, pre0, pre1);
                 }
                 const int ab = (int)(step & 1);
-                if (!wait_bar(&acc_full[ab], (uint32_t)((step >> 1) & 1), abort_flag, a.status)) {
-                    ok = false;
-                    break;
-                }
+                if (ok) ok = warp_wait(&acc_full[ab], (uint32_t)((step >> 1) & 1), abort_flag, a.status);
+                if (!ok) continue;
                 tc_fence_after();
                 float v[64];
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * kAccCols + half * 64);
@@ -461,13 +480,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ssum += s2.x + s2.y;
                 }
             }
-            if (!ok) break;
-            // merge the two column halves of each row, then write
+            // merge the two column halves of each row, then write (both halves always
+            // reach the named barrier, also after an abort)
             float2* mb = merge + (it & 1) * 128;
             if (half == 1) mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
                                                                 : make_float2(m, ssum);
             named_bar(1 + q, 64);
-            if (half == 0) {
+            if (half == 0 && ok) {
                 const float2 o = mb[q * 32 + lane];
                 if (MODE == kModeImp) {
                     const int j = t.fix_row0 + row;
@@ -486,9 +505,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1)
+    if (warp == 1) {
+        __syncwarp();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(2 * kAccCols));
+    }
 }
 
 // ------------------------------------------------------------------- host side
