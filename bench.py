@@ -104,11 +104,16 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ workload
-def workload_for_rank(rank: int):
+def workload_for_rank(rank: int, name: str | None = None, prompts: int = 0):
+    """The named workload (default: the Qwen2.5-7B varlen batch), optionally cut to
+    its first `prompts` prompts (same lengths and bytes as in the full batch: the
+    generator is counter-based); ranks > 0 draw their own batch of the same shape."""
+    import dataclasses
     from synth import workloads as W
-    w = W.C2
+    w = W.WORKLOADS[name] if name else W.C2
+    if prompts:
+        w = dataclasses.replace(w, B=min(prompts, w.B), name=f"{w.name}[:{min(prompts, w.B)}]")
     if rank:
-        import dataclasses
         w = dataclasses.replace(w, seed=w.seed + 1000 * rank)
     return w
 
@@ -207,7 +212,12 @@ def run_ours(args, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = workload_for_rank(rank)
+    w = workload_for_rank(rank, args.workload, args.prompts)
+    need = resident_bytes(w)
+    free = torch.cuda.mem_get_info(dev)[0]
+    if need > 0.85 * free:
+        raise SystemExit(f"{w.name}: {need / 2**30:.1f} GiB of resident inputs exceed the free "
+                         f"{free / 2**30:.1f} GiB; use --prompts to bench a slice of it")
     st = Step(estp, w, dev)
     torch.cuda.synchronize()
     n_layers = len(w.layers)
@@ -288,7 +298,7 @@ def run_ours(args, rank, world, local_rank):
     return {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "sum_tokens_per_gpu": st_tokens(w),
                    "seq_len": f"U[{w.T_lo},{w.T_hi}]", "vocab": w.V, "layers": len(w.layers),
                    "Hq": w.Hq, "Hkv": w.Hkv, "head_dim": w.d, "hidden": w.D,
@@ -298,6 +308,13 @@ def run_ours(args, rank, world, local_rank):
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": st_launches(w) * K, "clocks": clocks,
     }
+
+
+def resident_bytes(w):
+    sumT = int(w.cu_seqlens()[-1])
+    esz = 2 if w.dtype == "bf16" else 4
+    return (sumT * w.V * esz + len(w.layers) * sumT * (w.Hq + w.Hkv) * w.d * esz
+            + sumT * w.D * esz + w.Hq * sumT * 4)
 
 
 def st_tokens(w):
@@ -408,7 +425,7 @@ def cpu_baseline(w, seconds_hint):
 def run_reference(args, rank, world):
     if rank != 0:
         return None
-    w = workload_for_rank(0)
+    w = workload_for_rank(0, args.workload, args.prompts)
     vals = []
     desc, n = "", 1
     for i in range(args.warmup + args.steps):
@@ -431,12 +448,16 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="rough CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=None,
+                    help="workload name (default qwen2.5-7b_varlen16); see synth/workloads.py")
+    ap.add_argument("--prompts", type=int, default=0,
+                    help="bench only the first N prompts of the workload")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -17,8 +17,20 @@
 namespace estp {
 namespace {
 
+#ifndef ESTP_ENT_UNROLL
+#define ESTP_ENT_UNROLL 8
+#endif
+#ifndef ESTP_ENT_MINB
+#define ESTP_ENT_MINB 3
+#endif
+#ifndef ESTP_ENT_PACKED   // 1: packed f32x2 FMA/ADD; 0: scalar FMA/ADD
+#define ESTP_ENT_PACKED 0
+#endif
+#ifndef ESTP_ENT_PREFETCH // 1: next batch loaded while the current one is reduced
+#define ESTP_ENT_PREFETCH 0
+#endif
 constexpr int kEntThreads = 256;
-constexpr int kEntUnroll = 4;           // 16-byte loads in flight per lane
+constexpr int kEntUnroll = ESTP_ENT_UNROLL;  // 16-byte loads per lane per batch (two batches in flight)
 constexpr float kMaskedLogit = -1e30f;  // finite: 2^(masked - m) = 0 and 0 * d = 0
 
 struct EntPart {
@@ -98,70 +110,158 @@ __device__ __forceinline__ void mask_f32(uint4& v, int valid) {
         if (e >= valid) w[e] = __float_as_uint(kMaskedLogit);
 }
 
-// One lane's share of units [c0, c1) of one row: lane handles c0 + lane + 32k.
+// Loads the units c, c + 32, .. c + 32 (kEntUnroll - 1) of a row segment ending at c1;
+// units at or past c1 become masked logits (they contribute nothing).
+template <bool kBf16>
+__device__ __forceinline__ void load_batch(const char* row, int64_t c, int64_t c1, int64_t nvec,
+                                           int tail_valid, uint4* v) {
+    constexpr int kPerUnit = kBf16 ? 8 : 4;
+#pragma unroll
+    for (int k = 0; k < kEntUnroll; ++k) {
+        const int64_t ck = c + 32 * k;
+        if (ck < c1) {
+            v[k] = ld_stream(row + ck * 16);
+            if (ck == nvec - 1 && tail_valid < kPerUnit) {
+                if (kBf16) mask_bf16(v[k], tail_valid); else mask_f32(v[k], tail_valid);
+            }
+        } else if (kBf16) {
+            v[k] = make_uint4(0xF149F149u, 0xF149F149u, 0xF149F149u, 0xF149F149u);
+        } else {
+            const uint32_t n = __float_as_uint(kMaskedLogit);
+            v[k] = make_uint4(n, n, n, n);
+        }
+    }
+}
+
+// Folds one batch of kEntUnroll units into the lane's running (m, s, t): one max and
+// one rescale per batch, then two interleaved accumulator pairs to shorten the
+// dependent add chains.
+__device__ __forceinline__ void accum1(float x, float m, float& s, float& t) {
+    const float d = fmaf(x, kLog2e, -m);  // y - m
+    const float e = ex2(d);
+    s += e;
+    t = fmaf(e, d, t);
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void reduce_batch(const uint4* v, float& m, float2& s, float2& t,
+                                             float2& s1, float2& t1) {
+    float bm;
+    if (kBf16) {  // tree max over the batch's bf16 pairs
+        __nv_bfloat162 mx[kEntUnroll];
+#pragma unroll
+        for (int k = 0; k < kEntUnroll; ++k) {
+            const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v[k]);
+            mx[k] = __hmax2(__hmax2(p[0], p[1]), __hmax2(p[2], p[3]));
+        }
+#pragma unroll
+        for (int w = kEntUnroll / 2; w > 0; w >>= 1)
+#pragma unroll
+            for (int k = 0; k < w; ++k) mx[k] = __hmax2(mx[k], mx[k + w]);
+        bm = fmaxf(__low2float(mx[0]), __high2float(mx[0]));
+    } else {
+        float mx[kEntUnroll];
+#pragma unroll
+        for (int k = 0; k < kEntUnroll; ++k)
+            mx[k] = fmaxf(fmaxf(__uint_as_float(v[k].x), __uint_as_float(v[k].y)),
+                          fmaxf(__uint_as_float(v[k].z), __uint_as_float(v[k].w)));
+#pragma unroll
+        for (int w = kEntUnroll / 2; w > 0; w >>= 1)
+#pragma unroll
+            for (int k = 0; k < w; ++k) mx[k] = fmaxf(mx[k], mx[k + w]);
+        bm = mx[0];
+    }
+    const float new_m = fmaxf(m, bm * kLog2e);
+    const float dm = m - new_m;  // <= 0
+    const float f = ex2(dm);
+    t = make_float2(f * fmaf(dm, s.x, t.x), f * fmaf(dm, s.y, t.y));
+    t1 = make_float2(f * fmaf(dm, s1.x, t1.x), f * fmaf(dm, s1.y, t1.y));
+    s = make_float2(s.x * f, s.y * f);
+    s1 = make_float2(s1.x * f, s1.y * f);
+    m = new_m;
+#pragma unroll
+    for (int k = 0; k < kEntUnroll; ++k) {
+        if (ESTP_ENT_PACKED) {
+            if (kBf16) {
+                accum_pair(make_float2(bf16lo(v[k].x), bf16hi(v[k].x)), m, s, t);
+                accum_pair(make_float2(bf16lo(v[k].y), bf16hi(v[k].y)), m, s1, t1);
+                accum_pair(make_float2(bf16lo(v[k].z), bf16hi(v[k].z)), m, s, t);
+                accum_pair(make_float2(bf16lo(v[k].w), bf16hi(v[k].w)), m, s1, t1);
+            } else {
+                accum_pair(make_float2(__uint_as_float(v[k].x), __uint_as_float(v[k].y)), m, s, t);
+                accum_pair(make_float2(__uint_as_float(v[k].z), __uint_as_float(v[k].w)), m, s1, t1);
+            }
+        } else if (kBf16) {  // four independent (s, t) chains
+            accum1(bf16lo(v[k].x), m, s.x, t.x);
+            accum1(bf16hi(v[k].x), m, s.y, t.y);
+            accum1(bf16lo(v[k].y), m, s1.x, t1.x);
+            accum1(bf16hi(v[k].y), m, s1.y, t1.y);
+            accum1(bf16lo(v[k].z), m, s.x, t.x);
+            accum1(bf16hi(v[k].z), m, s.y, t.y);
+            accum1(bf16lo(v[k].w), m, s1.x, t1.x);
+            accum1(bf16hi(v[k].w), m, s1.y, t1.y);
+        } else {
+            accum1(__uint_as_float(v[k].x), m, s.x, t.x);
+            accum1(__uint_as_float(v[k].y), m, s.y, t.y);
+            accum1(__uint_as_float(v[k].z), m, s1.x, t1.x);
+            accum1(__uint_as_float(v[k].w), m, s1.y, t1.y);
+        }
+    }
+}
+
+// One lane's share of units [c0, c1) of one row (lane handles c0 + lane + 32k), with
+// the next batch's loads issued before the current batch is reduced.
+// One lane's share of units [c0, c1) of one row (lane handles c0 + lane + 32k).
+// Full batches run without bounds checks through a moving pointer; the ragged
+// remainder and the row's partial last unit (when V is not a multiple of the
+// unit width) go through the checked loader.
 template <bool kBf16>
 __device__ __forceinline__ void segment(const char* row, int64_t c0, int64_t c1, int64_t nvec,
                                         int tail_valid, float& m, float2& s, float2& t) {
     const int lane = threadIdx.x & 31;
     constexpr int kPerUnit = kBf16 ? 8 : 4;
-    for (int64_t c = c0 + lane; c < c1; c += 32 * kEntUnroll) {
-        uint4 v[kEntUnroll];
+    constexpr int64_t kStride = 32 * kEntUnroll;
+    float2 s1 = make_float2(0.f, 0.f), t1 = make_float2(0.f, 0.f);
+    // the unchecked range excludes a partial last unit of the row
+    const int64_t c1m = (c1 == nvec && tail_valid < kPerUnit) ? c1 - 1 : c1;
+    int64_t c = c0 + lane;
+    const uint4* p = reinterpret_cast<const uint4*>(row) + c;
+    if (ESTP_ENT_PREFETCH && c + kStride * 2 - 32 < c1m) {
+        uint4 va[kEntUnroll], vb[kEntUnroll];
 #pragma unroll
-        for (int k = 0; k < kEntUnroll; ++k) {
-            int64_t ck = c + 32 * k;
-            if (ck < c1) {
-                v[k] = ld_stream(row + ck * 16);
-                if (ck == nvec - 1 && tail_valid < kPerUnit) {
-                    if (kBf16) mask_bf16(v[k], tail_valid); else mask_f32(v[k], tail_valid);
-                }
-            } else {
-                if (kBf16) v[k] = make_uint4(0xF149F149u, 0xF149F149u, 0xF149F149u, 0xF149F149u);
-                else {
-                    uint32_t n = __float_as_uint(kMaskedLogit);
-                    v[k] = make_uint4(n, n, n, n);
-                }
+        for (int k = 0; k < kEntUnroll; ++k) va[k] = ld_stream(p + 32 * k);
+        while (true) {
+            p += kStride;
+            c += kStride;
+            const bool more = c + kStride - 32 < c1m;
+            if (more) {
+#pragma unroll
+                for (int k = 0; k < kEntUnroll; ++k) vb[k] = ld_stream(p + 32 * k);
             }
+            reduce_batch<kBf16>(va, m, s, t, s1, t1);
+            if (!more) break;
+#pragma unroll
+            for (int k = 0; k < kEntUnroll; ++k) va[k] = vb[k];
         }
-        // batch max (one rescale per batch of kEntUnroll units)
-        float bm;
-        if (kBf16) {
-            __nv_bfloat162 mx = *reinterpret_cast<__nv_bfloat162*>(&v[0].x);
+    } else {
+        for (; c + kStride - 32 < c1m; c += kStride, p += kStride) {
+            uint4 v[kEntUnroll];
 #pragma unroll
-            for (int k = 0; k < kEntUnroll; ++k) {
-                const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v[k]);
-#pragma unroll
-                for (int q = (k == 0 ? 1 : 0); q < 4; ++q) mx = __hmax2(mx, p[q]);
-            }
-            bm = fmaxf(__low2float(mx), __high2float(mx));
-        } else {
-            bm = __uint_as_float(v[0].x);
-#pragma unroll
-            for (int k = 0; k < kEntUnroll; ++k) {
-                bm = fmaxf(bm, __uint_as_float(v[k].x));
-                bm = fmaxf(bm, __uint_as_float(v[k].y));
-                bm = fmaxf(bm, __uint_as_float(v[k].z));
-                bm = fmaxf(bm, __uint_as_float(v[k].w));
-            }
-        }
-        float new_m = fmaxf(m, bm * kLog2e);
-        rescale(m, s, t, new_m);
-#pragma unroll
-        for (int k = 0; k < kEntUnroll; ++k) {
-            if (kBf16) {
-                accum_pair(make_float2(bf16lo(v[k].x), bf16hi(v[k].x)), m, s, t);
-                accum_pair(make_float2(bf16lo(v[k].y), bf16hi(v[k].y)), m, s, t);
-                accum_pair(make_float2(bf16lo(v[k].z), bf16hi(v[k].z)), m, s, t);
-                accum_pair(make_float2(bf16lo(v[k].w), bf16hi(v[k].w)), m, s, t);
-            } else {
-                accum_pair(make_float2(__uint_as_float(v[k].x), __uint_as_float(v[k].y)), m, s, t);
-                accum_pair(make_float2(__uint_as_float(v[k].z), __uint_as_float(v[k].w)), m, s, t);
-            }
+            for (int k = 0; k < kEntUnroll; ++k) v[k] = ld_stream(p + 32 * k);
+            reduce_batch<kBf16>(v, m, s, t, s1, t1);
         }
     }
+    if (c < c1) {  // remainder: fewer than kEntUnroll units left for this lane
+        uint4 v[kEntUnroll];
+        load_batch<kBf16>(row, c, c1, nvec, tail_valid, v);
+        reduce_batch<kBf16>(v, m, s, t, s1, t1);
+    }
+    s = make_float2(s.x + s1.x, s.y + s1.y);
+    t = make_float2(t.x + t1.x, t.y + t1.y);
 }
 
 template <bool kBf16>
-__global__ void __launch_bounds__(kEntThreads) entropy_kernel(EntArgs a) {
+__global__ void __launch_bounds__(kEntThreads, ESTP_ENT_MINB) entropy_kernel(EntArgs a) {
     const int lane = threadIdx.x & 31;
     const int64_t w = (int64_t)blockIdx.x * (kEntThreads / 32) + (threadIdx.x >> 5);
     if (w >= a.n_warps) return;

@@ -53,6 +53,7 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
         base[B] = ok ? sums[1023] : 0;
         info->ok = ok ? 1 : 0;
         info->total = ok ? sums[1023] : 0;
+        info->next = 0;
     }
     if (tid == 0 && !ok) report(status, ESTP_ERR_INVALID_ARG);
 }
@@ -142,7 +143,7 @@ __global__ void __launch_bounds__(kSThreads) lse_simt_kernel(SimtArgs a) {
     const int total = a.info->total;
     const int rep = a.Hq / a.Hkv;
     for (int item = blockIdx.x; item < total; item += gridDim.x) {
-        const LseItem it = decode_lse_item(item, a.base, a.B, a.cu, kSTile);
+        const LseItem it = decode_lse_item(item, a.base, a.B, a.cu, kSTile, a.hs.n_heads);
         const int h = a.hs.head_list[it.hslot];
         const int q0 = it.qt * kSTile;
         __syncthreads();

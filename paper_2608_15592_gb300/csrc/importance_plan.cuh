@@ -8,8 +8,9 @@
 //   f(nt) = sum_{m=1..nt} ceil(m / qc) = qc*a*(a+1)/2 + r*(a+1),  nt = a*qc + r,
 // and key tile kt starts at item F(kt) = f(nt) - f(nt - kt).
 //
-// LSE items: (head slot, query tile), the query tiles of a prompt numbered from
-// the last (longest rows) to the first.
+// LSE items: (query tile, head slot), numbered from the last query tile (longest
+// rows, most key tiles) to the first, so that a dynamic scheduler hands out the
+// largest items of a prompt first.
 #pragma once
 #include "estp_internal.cuh"
 
@@ -23,6 +24,8 @@ __host__ __device__ __forceinline__ int64_t items_f(int64_t n, int qc) {
 struct PlanInfo {
     int32_t ok;      // 1 when cu_seqlens passed the device checks
     int32_t total;   // total items
+    int32_t next;    // dynamic work counter of the persistent kernels (zeroed by the plan)
+    int32_t pad;
 };
 
 // Prefix of per-prompt item counts (base[B+1]) and validation.  One CTA of 1024.
@@ -69,15 +72,16 @@ struct LseItem {
 };
 
 __device__ __forceinline__ LseItem decode_lse_item(int item, const int32_t* base, int B,
-                                                   const int32_t* cu, int tile) {
+                                                   const int32_t* cu, int tile, int n_heads) {
     LseItem it;
     it.b = upper_slot(base, B, item);
     it.t0 = cu[it.b];
     it.T = cu[it.b + 1] - cu[it.b];
     const int nt = (it.T + tile - 1) / tile;
     const int local = item - base[it.b];
-    it.hslot = local / nt;
-    it.qt = nt - 1 - (local - it.hslot * nt);
+    const int rank = local / n_heads;
+    it.hslot = local - rank * n_heads;
+    it.qt = nt - 1 - rank;
     return it;
 }
 

@@ -23,6 +23,7 @@
 #include <cudaTypedefs.h>
 
 #include "importance_tc.cuh"
+#include "ptx.cuh"
 
 namespace estp {
 namespace {
@@ -32,7 +33,7 @@ constexpr int kQcTc = 4;
 constexpr int kThreads = 320;          // 10 warps
 constexpr int kEpiWarp0 = 2;           // warps 2..9
 constexpr int kAccCols = 128;
-constexpr long long kWaitCycles = 4000000000ll;
+constexpr int kSched = 4;              // depth of the item-index ring (producer -> consumers)
 
 enum Mode { kModeLse = 0, kModeImp = 1 };
 
@@ -48,9 +49,11 @@ struct Cfg {
     static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [8 warps][64] f32
     static constexpr int kMergeOff = kNlOff + 8 * 64 * 4;             // [2][4][32] float2
     static constexpr int kBarOff = kMergeOff + 2 * 4 * 32 * 8;
-    static constexpr int kNumBars = 2 + 2 + 2 * kStages + 2 + 2 + 1;
-    static constexpr int kMiscOff = kBarOff + kNumBars * 8;           // tmem addr, abort flag
-    static constexpr int kSmemBytes = kMiscOff + 16 + 1024;          // + alignment slack
+    // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[2], drain,
+    // sched_full/empty[kSched], xfull/xempty[2][4]
+    static constexpr int kNumBars = 2 + 2 + 2 * kStages + 2 + 2 + 1 + 2 * kSched + 16;
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
+    static constexpr int kSmemBytes = kMiscOff + 16 + 4 * kSched + 1024;  // + alignment slack
 };
 
 struct TcArgs {
@@ -69,75 +72,6 @@ struct TcArgs {
 };
 
 // ------------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-                 "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Bounded wait: false (and the CTA's abort flag set) when the barrier does not
-// complete in time or another role has already aborted.
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status) {
-    if (*abort_flag) return false;
-    if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (!mbar_try_wait(bar, parity)) {
-        if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitCycles) {
-            *abort_flag = 1;
-            report(status, ESTP_ERR_TIMEOUT);
-            return false;
-        }
-    }
-    return true;
-}
-
-// Bounded wait that ignores the abort flag (used to drain outstanding MMAs).
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* status) {
-    const long long t0 = clock64();
-    while (!mbar_try_wait(bar, parity)) {
-        if (clock64() - t0 > kWaitCycles) {
-            report(status, ESTP_ERR_TIMEOUT);
-            return;
-        }
-    }
-}
-
-// Warp-uniform bounded wait: lane 0 polls, every lane gets the same answer.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
-    bool r = false;
-    if ((threadIdx.x & 31) == 0) r = wait_bar(bar, parity, abort_flag, status);
-    r = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0;
-    __syncwarp();
-    return r;
-}
-
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
                                             uint64_t* bar) {
     asm volatile(
@@ -203,9 +137,6 @@ __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ void named_bar(int id, int n) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
-}
 
 // --------------------------------------------------------------- item description
 struct TcItem {
@@ -221,7 +152,7 @@ template <int MODE>
 __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
     TcItem t;
     if (MODE == kModeLse) {
-        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kTile);
+        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kTile, a.hs.n_heads);
         t.b = li.b; t.T = li.T; t.t0 = li.t0;
         t.h = a.hs.head_list[li.hslot];
         t.fix_y = t.h;
@@ -282,8 +213,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* acc_full = bars + 4 + 2 * C::kStages;
     uint64_t* acc_empty = acc_full + 2;
     uint64_t* drain = acc_empty + 2;
+    uint64_t* sched_full = drain + 1;             // [kSched]
+    uint64_t* sched_empty = sched_full + kSched;  // [kSched]
+    uint64_t* xfull = sched_empty + kSched;       // [2][4]: half-1 partials ready
+    uint64_t* xempty = xfull + 8;                 // [2][4]: half-0 has read them
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 4);
+    volatile int* sched_item = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 16);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -298,8 +234,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&ring_empty[i], 1);
         }
         mbar_init(drain, 1);
+        for (int i = 0; i < kSched; ++i) {
+            mbar_init(&sched_full[i], 1);
+            mbar_init(&sched_empty[i], 1 + 8);  // MMA thread + 8 epilogue warps
+        }
+        for (int i = 0; i < 8; ++i) {
+            mbar_init(&xfull[i], 1);
+            mbar_init(&xempty[i], 1);
+        }
         *abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_fence_init();
     }
     if (warp == 1) {  // TMEM: 2 accumulators x 128 columns
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -311,16 +255,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const int total = a.info->total;
+    PlanInfo* info = const_cast<PlanInfo*>(a.info);
+    const int total = info->total;
+
+    // Item k of this CTA, published by the producer in slot k % kSched (-1 = no more).
+    auto consume_item = [&](int k, bool warp_uniform) -> int {
+        const int slot = k % kSched;
+        const uint32_t par = (uint32_t)((k / kSched) & 1);
+        bool got;
+        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
+        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
+        if (!got) return -1;
+        const int item = sched_item[slot];
+        if (warp_uniform) __syncwarp();
+        if (!warp_uniform || lane == 0) mbar_arrive(&sched_empty[slot]);
+        return item;
+    };
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_fix)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_str)) : "memory");
-            int it = 0;
             long long step = 0;
-            for (int item = blockIdx.x; item < total; item += gridDim.x, ++it) {
+            int item = blockIdx.x;
+            for (int it = 0;; ++it) {
+                if (item >= total) item = -1;
+                const int slot = it % kSched;
+                if (it >= kSched &&
+                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
+                    break;
+                sched_item[slot] = item;
+                mbar_arrive(&sched_full[slot]);  // release: the item index is visible to waiters
+                if (item < 0) break;
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
@@ -346,15 +313,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     (int)(t.t0 + row0), &ring_full[stage]);
                 }
                 if (!ok) break;
+                item = (int)gridDim.x + atomicAdd(&info->next, 1);
             }
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            int it = 0;
             long long step = 0;
             bool issued = false;
-            for (int item = blockIdx.x; item < total; item += gridDim.x, ++it) {
+            for (int it = 0;; ++it) {
+                const int item = consume_item(it, false);
+                if (item < 0) break;
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
@@ -397,9 +366,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = q * 32 + lane;             // accumulator row owned by this thread
         float* nl = nl_all + (warp - kEpiWarp0) * 64;
         long long step = 0;
-        int it = 0;
-        bool ok = true;  // false once any wait gave up: the loops then run without waiting
-        for (int item = blockIdx.x; item < total; item += gridDim.x, ++it) {
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            const int item = consume_item(it, true);
+            if (item < 0) break;
             const TcItem t = make_item<MODE>(a, item);
             float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
             float m = -1e30f, ssum = 0.f;          // LSE mode
@@ -413,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 r1 = i1 < t.T ? -l[i1] * kLog2e : -INFINITY;
             };
             if (MODE == kModeImp) load_nl(0, pre0, pre1);
-            for (int s = 0; s < t.n_steps; ++s, ++step) {
+            for (int s = 0; s < t.n_steps && ok; ++s, ++step) {
                 int y, row0, head, qt;
                 step_tile<MODE>(a, t, s, y, row0, head, qt);
                 if (MODE == kModeImp) {
@@ -424,8 +394,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (s + 1 < t.n_steps) load_nl(s + 1, pre0, pre1);
                 }
                 const int ab = (int)(step & 1);
-                if (ok) ok = warp_wait(&acc_full[ab], (uint32_t)((step >> 1) & 1), abort_flag, a.status);
-                if (!ok) continue;
+                ok = warp_wait(&acc_full[ab], (uint32_t)((step >> 1) & 1), abort_flag, a.status);
+                if (!ok) break;
                 tc_fence_after();
                 float v[64];
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * kAccCols + half * 64);
@@ -480,14 +450,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ssum += s2.x + s2.y;
                 }
             }
-            // merge the two column halves of each row, then write (both halves always
-            // reach the named barrier, also after an abort)
-            float2* mb = merge + (it & 1) * 128;
-            if (half == 1) mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
-                                                                : make_float2(m, ssum);
-            named_bar(1 + q, 64);
-            if (half == 0 && ok) {
+            if (!ok) break;
+            // merge the two column halves of each row (bounded mbarrier hand-off), then write
+            const int pb = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            float2* mb = merge + pb * 128;
+            uint64_t* xf = &xfull[pb * 4 + q];
+            uint64_t* xe = &xempty[pb * 4 + q];
+            if (half == 1) {
+                if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status);
+                if (!ok) break;
+                mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
+                                                     : make_float2(m, ssum);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(xf);
+            } else {
+                ok = warp_wait(xf, use & 1, abort_flag, a.status);
+                if (!ok) break;
                 const float2 o = mb[q * 32 + lane];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(xe);
                 if (MODE == kModeImp) {
                     const int j = t.fix_row0 + row;
                     if (j < t.T)
