@@ -33,8 +33,7 @@ constexpr int kQcTc = 4;
 constexpr int kThreads = 320;          // 10 warps
 constexpr int kEpiWarp0 = 2;           // warps 2..9
 constexpr int kAccCols = 128;
-constexpr int kSched = 4;              // depth of the item ring (producer -> consumers)
-constexpr int kPlanCache = 2048;       // prompts whose plan and offsets are cached in smem
+constexpr int kSched = 4;              // depth of the item-index ring (producer -> consumers)
 
 enum Mode { kModeLse = 0, kModeImp = 1 };
 
@@ -54,9 +53,7 @@ struct Cfg {
     // sched_full/empty[kSched], xfull/xempty[2][4]
     static constexpr int kNumBars = 2 + 2 + 2 * kStages + 2 + 2 + 1 + 2 * kSched + 16;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
-    static constexpr int kItemOff = kMiscOff + 16;                     // [kSched] decoded items
-    static constexpr int kPlanOff = kItemOff + kSched * 64;            // cached base[], cu[]
-    static constexpr int kSmemBytes = kPlanOff + 2 * 4 * (kPlanCache + 1) + 1024;  // + alignment slack
+    static constexpr int kSmemBytes = kMiscOff + 16 + 4 * kSched + 1024;  // + alignment slack
 };
 
 struct TcArgs {
@@ -143,7 +140,6 @@ __device__ __forceinline__ void tmem_wait_ld() {
 
 // --------------------------------------------------------------- item description
 struct TcItem {
-    int valid;
     int b, T;
     int64_t t0;
     int fix_y, fix_row0;       // fixed tile: head (LSE: query head, IMP: KV head), first row
@@ -152,15 +148,11 @@ struct TcItem {
     int h, g, kt, qt0, qt1, chunk;
 };
 
-static_assert(sizeof(TcItem) <= 64, "a decoded item fills one 64-byte ring slot");
-
 template <int MODE>
-__device__ __forceinline__ TcItem make_item(const TcArgs& a, int item, const int32_t* base,
-                                            const int32_t* cu) {
+__device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
     TcItem t;
-    t.valid = 1;
     if (MODE == kModeLse) {
-        const LseItem li = decode_lse_item(item, base, a.B, cu, kTile, a.hs.n_heads);
+        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kTile, a.hs.n_heads);
         t.b = li.b; t.T = li.T; t.t0 = li.t0;
         t.h = a.hs.head_list[li.hslot];
         t.fix_y = t.h;
@@ -169,7 +161,7 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item, const int
         t.n_steps = li.qt + 1;  // key tiles 0..qt
         t.g = 0; t.kt = 0; t.qt1 = li.qt + 1; t.chunk = 0;
     } else {
-        const ImpItem ii = decode_imp_item(item, base, a.B, cu, kTile, kQcTc);
+        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kTile, kQcTc);
         t.b = ii.b; t.T = ii.T; t.t0 = ii.t0;
         t.g = ii.g; t.kt = ii.kt; t.qt0 = ii.qt0; t.qt1 = ii.qt1;
         t.chunk = (ii.qt0 - ii.kt) / kQcTc;
@@ -227,9 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* xempty = xfull + 8;                 // [2][4]: half-0 has read them
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 4);
-    TcItem* sched_item = reinterpret_cast<TcItem*>(sm + C::kItemOff);
-    int32_t* base_s = reinterpret_cast<int32_t*>(sm + C::kPlanOff);
-    int32_t* cu_s = base_s + (kPlanCache + 1);
+    volatile int* sched_item = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 16);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -267,31 +257,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
     PlanInfo* info = const_cast<PlanInfo*>(a.info);
     const int total = info->total;
-    // the producer decodes items from a shared-memory copy of the plan when it fits
-    const bool cached = a.B <= kPlanCache;
-    if (warp == 0 && cached)
-        for (int i = lane; i <= a.B; i += 32) {
-            base_s[i] = a.base[i];
-            cu_s[i] = a.cu[i];
-        }
-    __syncwarp();
-    const int32_t* base_p = cached ? base_s : a.base;
-    const int32_t* cu_p = cached ? cu_s : a.cu;
 
-    // Item k of this CTA, decoded by the producer into slot k % kSched (valid = 0: no more).
-    auto consume_item = [&](int k, bool warp_uniform) -> TcItem {
+    // Item k of this CTA, published by the producer in slot k % kSched (-1 = no more).
+    auto consume_item = [&](int k, bool warp_uniform) -> int {
         const int slot = k % kSched;
         const uint32_t par = (uint32_t)((k / kSched) & 1);
         bool got;
         if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
         else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
-        TcItem t;
-        t.valid = 0;
-        if (!got) return t;
-        t = sched_item[slot];
+        if (!got) return -1;
+        const int item = sched_item[slot];
         if (warp_uniform) __syncwarp();
         if (!warp_uniform || lane == 0) mbar_arrive(&sched_empty[slot]);
-        return t;
+        return item;
     };
 
     if (warp == 0) {
@@ -307,12 +285,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (it >= kSched &&
                     !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
                     break;
-                TcItem t;
-                t.valid = 0;
-                if (item >= 0) t = make_item<MODE>(a, item, base_p, cu_p);
-                sched_item[slot] = t;
-                mbar_arrive(&sched_full[slot]);  // release: the item is visible to waiters
+                sched_item[slot] = item;
+                mbar_arrive(&sched_full[slot]);  // release: the item index is visible to waiters
                 if (item < 0) break;
+                const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
                 mbar_expect_tx(&fix_full[fb], C::kTileBytes);
@@ -346,8 +322,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long step = 0;
             bool issued = false;
             for (int it = 0;; ++it) {
-                const TcItem t = consume_item(it, false);
-                if (!t.valid) break;
+                const int item = consume_item(it, false);
+                if (item < 0) break;
+                const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
                 const uint32_t fix_addr = smem_u32(fix + fb * C::kTileBytes);
@@ -391,8 +368,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         long long step = 0;
         bool ok = true;
         for (int it = 0; ok; ++it) {
-            const TcItem t = consume_item(it, true);
-            if (!t.valid) break;
+            const int item = consume_item(it, true);
+            if (item < 0) break;
+            const TcItem t = make_item<MODE>(a, item);
             float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
             float m = -1e30f, ssum = 0.f;          // LSE mode
             float pre0 = 0.f, pre1 = 0.f;
