@@ -89,6 +89,26 @@ estp_status estp_token_entropy(estp_ctx* ctx, const void* logits, estp_dtype dty
                                const int32_t* cu_seqlens, int32_t B, float* entropy_out,
                                estp_stream_t stream);
 
+/* Allocation-free token entropy.  The paper has no counterpart: this is a deployment
+ * variant of estp_token_entropy for callers that cannot allocate device memory, such
+ * as a serving engine whose allocator already owns all of HBM for its KV cache, or
+ * code running where cudaMalloc is not allowed.  It computes the same entropy_out as
+ * estp_token_entropy (same arguments, minus context and cu_seqlens) on the calling
+ * thread's current device, allocating nothing: its scratch (per-piece (max, sum,
+ * weighted sum) partials) is one file-scope static device array of 128 KiB (4096
+ * partial pairs) that every GPU loading this library holds until the process exits.
+ *   - The first call on a device looks up that array's device address (a one-time
+ *     set-up); make the first call before any stream capture.
+ *   - All calls share the array, and it keeps the last call's contents: calls that
+ *     overlap on the GPU (different streams, or concurrent host threads) race on it.
+ *     Order them on one stream.
+ *   - A GPU whose launch would need more than 4096 partial pairs (more than ~170 SMs
+ *     at the kernel's occupancy) gets ESTP_ERR_WORKSPACE and nothing is enqueued.
+ * Errors are reported as for estp_token_entropy; there is no device status word. */
+estp_status estp_token_entropy_noalloc(const void* logits, estp_dtype dtype, int64_t n_rows,
+                                       int64_t V, int64_t ld, float* entropy_out,
+                                       estp_stream_t stream);
+
 /* ------------------------------------------------------------------ (b)
  * Attention layout for one layer (Sec. 3.1): Q is [sumT, Hq, head_dim] and K is
  * [sumT, Hkv, head_dim], row-major and contiguous, dtype ESTP_BF16 or ESTP_F32.

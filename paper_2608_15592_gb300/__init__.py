@@ -32,7 +32,7 @@ ESTP_IMP_EXCLUDE_SELF = 1
 # every entry point declared in include/estp.h
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
-           "estp_attn_importance_finalize", "estp_pool")
+           "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc")
 
 
 class EstpError(RuntimeError):
@@ -70,6 +70,7 @@ def _load():
         "estp_attn_importance": ([P, P, P, ctypes.c_int, P, I32, I32, I32, F, P, I32, P, I32,
                                   I64, I32, ctypes.c_int, U32, P], ctypes.c_int),
         "estp_attn_importance_finalize": ([P, I32, P, P], ctypes.c_int),
+        "estp_token_entropy_noalloc": ([P, ctypes.c_int, I64, I64, I64, P, P], ctypes.c_int),
         "estp_pool": ([P, P, ctypes.c_int, I64, I64, P, P, P, I32, I64, MixParams,
                        ctypes.POINTER(_Head), P, P, P], ctypes.c_int),
     }

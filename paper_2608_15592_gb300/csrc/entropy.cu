@@ -12,6 +12,8 @@
 // bytes whatever V and n_rows are.  A warp finishes the rows it covers whole; a row
 // cut between warps leaves (m, s, t) partials that a second kernel merges in warp
 // order (deterministic).
+#include <mutex>
+
 #include "estp_internal.cuh"
 
 namespace estp {
@@ -347,4 +349,95 @@ estp_status launch_entropy(estp_ctx* ctx, const void* logits, estp_dtype dtype, 
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "entropy launch");
 }
 
+// ------------------------------------------------ allocation-free variant
+// Token entropy for callers that cannot allocate device memory: a serving engine whose
+// allocator already owns all of HBM (for its KV cache), or code running where
+// cudaMalloc is not allowed.  The per-piece partials that estp_token_entropy keeps in
+// the context workspace live here in one file-scope device array instead, so this path
+// needs no context and allocates nothing.  Every call shares the array: calls that
+// overlap on the GPU race on it.  No slot needs clearing: each is written before it is
+// read within a call.
+constexpr int64_t kNoAllocPieces = 4096;  // partial pairs the static scratch holds (128 KiB)
+static __device__ __align__(256) EntPart g_noalloc_part[2 * kNoAllocPieces];
+
+namespace {
+struct NoAllocDevice {
+    bool ready = false;
+    EntPart* part = nullptr;  // device address of g_noalloc_part on this device
+    int num_sms = 0;
+};
+std::mutex g_noalloc_mu;
+NoAllocDevice g_noalloc_devices[64];
+}  // namespace
+
+// Once per device, with that device current: the device address of the static scratch
+// (the host-side name g_noalloc_part is only a stand-in) and the SM count.
+static estp_status noalloc_setup(int dev, NoAllocDevice* out) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (dev < 0 || dev >= 64) return fail(ESTP_ERR_UNSUPPORTED, "device ordinal %d >= 64", dev);
+    NoAllocDevice& d = g_noalloc_devices[dev];
+    if (!d.ready) {
+        void* p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_part);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(entropy scratch)");
+        e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        d.part = static_cast<EntPart*>(p);
+        d.ready = true;
+    }
+    *out = d;
+    return ESTP_OK;
+}
+
+estp_status launch_entropy_noalloc(const void* logits, estp_dtype dtype, int64_t n_rows, int64_t V,
+                                   int64_t ld, float* H, cudaStream_t st) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    NoAllocDevice d;
+    estp_status s = noalloc_setup(dev, &d);
+    if (s != ESTP_OK) return s;
+    const int per_unit = dtype == ESTP_BF16 ? 8 : 4;
+    EntArgs a;
+    a.base = static_cast<const char*>(logits);
+    a.ld_bytes = ld * esize(dtype);
+    a.nvec = (V + per_unit - 1) / per_unit;
+    a.V = V;
+    a.units = n_rows * a.nvec;
+    int occ = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &occ, dtype == ESTP_BF16 ? entropy_kernel<true> : entropy_kernel<false>, kEntThreads, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
+    const int64_t max_warps = (int64_t)d.num_sms * (occ > 0 ? occ : 1) * (kEntThreads / 32);
+    a.n_warps = a.units < max_warps ? a.units : max_warps;
+    if (a.n_warps > kNoAllocPieces)
+        return fail(ESTP_ERR_WORKSPACE,
+                    "allocation-free entropy needs %lld partial pairs; its static scratch holds %lld",
+                    (long long)a.n_warps, (long long)kNoAllocPieces);
+    a.part = d.part;
+    a.H = H;
+    const int64_t blocks = (a.n_warps + kEntThreads / 32 - 1) / (kEntThreads / 32);
+    if (dtype == ESTP_BF16) entropy_kernel<true><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
+    else entropy_kernel<false><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
+    const int64_t mblocks = (n_rows + 255) / 256;
+    entropy_merge_kernel<<<(unsigned)mblocks, 256, 0, st>>>(a, n_rows, nullptr, 0, nullptr);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "entropy launch");
+}
+
 }  // namespace estp
+
+extern "C" estp_status estp_token_entropy_noalloc(const void* logits, estp_dtype dtype,
+                                                  int64_t n_rows, int64_t V, int64_t ld,
+                                                  float* entropy_out, estp_stream_t stream) {
+    using namespace estp;
+    if (dtype != ESTP_F32 && dtype != ESTP_BF16) return fail(ESTP_ERR_INVALID_ARG, "dtype");
+    if (n_rows < 0 || V < 1 || ld < V)
+        return fail(ESTP_ERR_INVALID_ARG, "need n_rows >= 0, V >= 1, ld >= V");
+    if (n_rows == 0) return ESTP_OK;
+    if (!logits || !entropy_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    if (!aligned16(logits) || (ld * esize(dtype)) % 16)
+        return fail(ESTP_ERR_INVALID_ARG, "logits base and row stride must be 16-byte aligned");
+    return launch_entropy_noalloc(logits, dtype, n_rows, V, ld, entropy_out,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
