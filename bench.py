@@ -118,6 +118,21 @@ def workload_for_rank(rank: int, name: str | None = None, prompts: int = 0):
     return w
 
 
+def aggregate_ranks(ms: float, tokens: float, device=None):
+    """Whole-job numbers from per-rank ones: the slowest rank's time (MAX) and the
+    tokens of all ranks (SUM).  Prompts are independent, so this is the only
+    cross-rank exchange; with one process it returns its inputs."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms, tokens
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    n = torch.tensor([tokens], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(n.item())
+
+
 def algorithmic(w, cu):
     """Per-launch algorithmic work of each kernel of one step."""
     import numpy as np
@@ -247,16 +262,7 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         torch.distributed.barrier()
     st.ctx.sync_status()
-    ms = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-        n = torch.tensor([float(st.sumT)], device=dev)
-        torch.distributed.all_reduce(n)
-        tokens = float(n.item())
-    else:
-        tokens = float(st.sumT)
+    ms, tokens = aggregate_ranks(start.elapsed_time(end), float(st.sumT), dev)
     ms_per_step = ms / K
     value = tokens * K / (ms / 1e3)
 
@@ -362,12 +368,8 @@ def run_e2e(args, st, estp, dev, world):
         step()
     b.record()
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    return {"value": st.sumT * world * K / (ms / 1e3), "unit": UNIT,
+    ms, tokens = aggregate_ranks(a.elapsed_time(b), float(st.sumT), dev)
+    return {"value": tokens * K / (ms / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": K}
 
 

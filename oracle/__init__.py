@@ -8,6 +8,7 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   token_entropy   Eq. 2-1 (Sec. 3.2)
   attn_lse        the row normaliser of the causal softmax A (Sec. 3.1)
   attn_colsum     sum_i A_ij of Eq. 2-0 for one layer, summed over query heads
+  attn_colsum_rows  the same from the rows i >= row_from only (exact for late keys)
   importance      Eq. 2-0: S_j = C_j / (N * layers * heads)
   pool            Eqs. 2-2, 2-3, 2-4
   length_head     Eq. 3-2 with a linear projection
@@ -52,6 +53,7 @@ class _Lib:
             "oracle_token_entropy": [P, I, I64, I64, I64, P, I],
             "oracle_attn_lse": [P, P, I, I, I, I, D, P, I, P, I],
             "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
+            "oracle_attn_colsum_rows": [P, P, I, I, I, I, D, P, I, P, I, I, I64, P, I],
             "oracle_importance": [P, P, I, I, I, P],
             "oracle_pool": [P, I, I64, I64, P, P, P, I, D, D, D, P, P],
             "oracle_length_head": [P, I, I64, P, P, P, I, P, P],
@@ -169,6 +171,24 @@ def attn_colsum(Q, K, cu_seqlens, scale, heads=None, exclude_self=False,
                                       float(scale), _ptr(h), nh, _ptr(cu), len(cu) - 1,
                                       int(bool(exclude_self)), _ptr(out), n_threads),
            "attn_colsum")
+    return out
+
+
+def attn_colsum_rows(Q, K, cu_seqlens, scale, row_from: int, heads=None, exclude_self=False,
+                     out: np.ndarray | None = None, n_threads: int = 0) -> np.ndarray:
+    """attn_colsum formed from the rows i >= row_from of every prompt: exact for keys
+    with prompt-local index >= row_from."""
+    Q, K, cu = np.ascontiguousarray(Q), np.ascontiguousarray(K), _cu(cu_seqlens)
+    sumT, Hq, d = Q.shape
+    Hkv = K.shape[1]
+    if out is None:
+        out = np.zeros(sumT, dtype=np.float64)
+    h = None if heads is None else np.ascontiguousarray(heads, dtype=np.int32)
+    nh = Hq if h is None else len(h)
+    _check(_load().oracle_attn_colsum_rows(_ptr(Q), _ptr(K), _dtype_code(Q), Hq, Hkv, d,
+                                           float(scale), _ptr(h), nh, _ptr(cu), len(cu) - 1,
+                                           int(bool(exclude_self)), int(row_from), _ptr(out),
+                                           n_threads), "attn_colsum_rows")
     return out
 
 

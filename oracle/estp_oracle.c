@@ -140,6 +140,7 @@ typedef struct {
     int64_t sumT;
     int64_t out_ld;   /* colsum: row length of the private buffers */
     int want_lse;
+    int64_t row_from; /* first prompt-local query row formed */
 } attn_ctx;
 
 static void attn_unit(void* vctx, int64_t unit, double* scratch) {
@@ -156,11 +157,12 @@ static void attn_unit(void* vctx, int64_t unit, double* scratch) {
     double* s = scratch; /* scores of one row, length >= T */
     for (int64_t t = 0; t < T; ++t)
         for (int x = 0; x < d; ++x) {
-            q[t * d + x] = load_elem(c->Q, c->dtype, ((t0 + t) * c->Hq + h) * (int64_t)d + x);
+            if (t >= c->row_from)  /* query rows before row_from are never formed */
+                q[t * d + x] = load_elem(c->Q, c->dtype, ((t0 + t) * c->Hq + h) * (int64_t)d + x);
             k[t * d + x] = load_elem(c->K, c->dtype, ((t0 + t) * c->Hkv + g) * (int64_t)d + x);
         }
     double* col = c->want_lse ? NULL : c->out + unit * c->out_ld;
-    for (int64_t i = 0; i < T; ++i) {
+    for (int64_t i = c->row_from; i < T; ++i) {
         /* s_ij = scale * q_i . k_j for the causal keys j <= i of the same prompt */
         double m = -INFINITY;
         for (int64_t j = 0; j <= i; ++j) {
@@ -201,15 +203,16 @@ int oracle_attn_lse(const void* Q, const void* K, int dtype, int Hq, int Hkv, in
     if (sumT == 0) return 0;
     if (!Q || !K || !lse_out) return -1;
     attn_ctx c = {Q, K, dtype, Hq, Hkv, d, scale, NULL, Hq, cu_seqlens, B, 0,
-                  lse_out, sumT, 0, 1};
+                  lse_out, sumT, 0, 1, 0};
     parallel_units(attn_unit, &c, (int64_t)B * Hq, (size_t)max_len(cu_seqlens, B), n_threads);
     return 0;
 }
 
-int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
-                       double scale, const int32_t* heads, int n_heads,
-                       const int32_t* cu_seqlens, int B, int exclude_self, double* C_out,
-                       int n_threads) {
+int oracle_attn_colsum_rows(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
+                            double scale, const int32_t* heads, int n_heads,
+                            const int32_t* cu_seqlens, int B, int exclude_self,
+                            int64_t row_from, double* C_out, int n_threads) {
+    if (row_from < 0) return -1;
     if (!valid_dtype(dtype) || Hq <= 0 || Hkv <= 0 || Hq % Hkv || d <= 0) return -1;
     if (!valid_cu(cu_seqlens, B)) return -1;
     if (heads) {
@@ -229,7 +232,7 @@ int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv,
     double* priv = (double*)calloc((size_t)(n_units * Tmax), sizeof(double));
     if (!priv) return -1;
     attn_ctx c = {Q, K, dtype, Hq, Hkv, d, scale, heads, n_heads, cu_seqlens, B,
-                  exclude_self, priv, sumT, Tmax, 0};
+                  exclude_self, priv, sumT, Tmax, 0, row_from};
     parallel_units(attn_unit, &c, n_units, (size_t)Tmax, n_threads);
     for (int b = 0; b < B; ++b) {
         int64_t t0 = cu_seqlens[b], T = (int64_t)cu_seqlens[b + 1] - cu_seqlens[b];
@@ -240,6 +243,14 @@ int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv,
     }
     free(priv);
     return 0;
+}
+
+int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
+                       double scale, const int32_t* heads, int n_heads,
+                       const int32_t* cu_seqlens, int B, int exclude_self, double* C_out,
+                       int n_threads) {
+    return oracle_attn_colsum_rows(Q, K, dtype, Hq, Hkv, d, scale, heads, n_heads, cu_seqlens, B,
+                                   exclude_self, 0, C_out, n_threads);
 }
 
 /* ------------------------------------------------------------ Eq. 2-0 */

@@ -58,6 +58,15 @@ int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv,
                        const int32_t* cu_seqlens, int B, int exclude_self, double* C_out,
                        int n_threads);
 
+/* The same column sums formed from the rows i >= row_from (prompt-local index) only.
+ * C_j depends only on rows i >= j, so C_out[j] is exact for every key j with local
+ * index >= row_from; smaller j receive only part of their mass.  Used to check late
+ * keys of prompts too long for the full O(T^2) evaluation. */
+int oracle_attn_colsum_rows(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
+                            double scale, const int32_t* heads, int n_heads,
+                            const int32_t* cu_seqlens, int B, int exclude_self,
+                            int64_t row_from, double* C_out, int n_threads);
+
 /* Eq. 2-0 with the head/layer mean: S_j = C_j / (N_b * n_layers * n_heads), where
  * N_b is the length of the prompt that holds token j.  S_out: [sumT]. */
 int oracle_importance(const double* C, const int32_t* cu_seqlens, int B, int n_layers,

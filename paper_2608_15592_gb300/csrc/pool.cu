@@ -214,30 +214,50 @@ __global__ void __launch_bounds__(kMergeThreads) pool_merge_kernel(const float* 
     }
 }
 
-// Linear head + softmax over K bins + expectation (Eq. 3-2).  One CTA per prompt.
-__global__ void __launch_bounds__(256) head_kernel(const float* pooled, int64_t D, const float* W,
-                                                   const float* bias, const float* centers, int K,
-                                                   float* pred) {
+// Linear head + softmax over K bins + expectation (Eq. 3-2).  One CTA of 32 warps per
+// prompt; warp w forms the logits z_k = W_k . h + bias_k of bins k = w, w + 32, ...
+// (float4 loads when rows are 16-byte aligned), then the CTA reduces the softmax and
+// the expectation in a fixed order.
+__global__ void __launch_bounds__(1024) head_kernel(const float* pooled, int64_t D, const float* W,
+                                                    const float* bias, const float* centers, int K,
+                                                    int vec4, float* pred) {
     __shared__ float z_s[1024];
     __shared__ float sh[32];
     const int b = blockIdx.x;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const float* h = pooled + (int64_t)b * D;
-    for (int k = wid; k < K; k += 8) {
+    for (int k = wid; k < K; k += 32) {
         const float* w = W + (int64_t)k * D;
-        float acc = 0.f;
-        for (int64_t x = lane; x < D; x += 32) acc = fmaf(w[x], h[x], acc);
+        float acc0 = 0.f, acc1 = 0.f;
+        if (vec4) {
+            const float4* w4 = reinterpret_cast<const float4*>(w);
+            const float4* h4 = reinterpret_cast<const float4*>(h);
+            const int64_t n4 = D / 4;
+            int64_t x = lane;
+            for (; x + 32 < n4; x += 64) {
+                const float4 a0 = w4[x], b0 = h4[x], a1 = w4[x + 32], b1 = h4[x + 32];
+                acc0 = fmaf(a0.x, b0.x, fmaf(a0.y, b0.y, fmaf(a0.z, b0.z, fmaf(a0.w, b0.w, acc0))));
+                acc1 = fmaf(a1.x, b1.x, fmaf(a1.y, b1.y, fmaf(a1.z, b1.z, fmaf(a1.w, b1.w, acc1))));
+            }
+            for (; x < n4; x += 32) {
+                const float4 a0 = w4[x], b0 = h4[x];
+                acc0 = fmaf(a0.x, b0.x, fmaf(a0.y, b0.y, fmaf(a0.z, b0.z, fmaf(a0.w, b0.w, acc0))));
+            }
+        } else {
+            for (int64_t x = lane; x < D; x += 32) acc0 = fmaf(w[x], h[x], acc0);
+        }
+        float acc = acc0 + acc1;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
         if (lane == 0) z_s[k] = acc + (bias ? bias[k] : 0.f);
     }
     __syncthreads();
     float mx = -INFINITY;
-    for (int k = threadIdx.x; k < K; k += 256) mx = fmaxf(mx, z_s[k]);
+    for (int k = threadIdx.x; k < K; k += 1024) mx = fmaxf(mx, z_s[k]);
     mx = block_reduce(mx, true, sh);
     float zs = 0.f, ys = 0.f;
-    for (int k = threadIdx.x; k < K; k += 256) {
-        float e = ex2((z_s[k] - mx) * kLog2e);
+    for (int k = threadIdx.x; k < K; k += 1024) {
+        const float e = ex2((z_s[k] - mx) * kLog2e);
         zs += e;
         ys = fmaf(e, centers[k], ys);
     }
@@ -283,8 +303,11 @@ estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int
     }
     dim3 mgrid((unsigned)B, (unsigned)((D + 4 * kMergeThreads - 1) / (4 * kMergeThreads)));
     pool_merge_kernel<<<mgrid, kMergeThreads, 0, st>>>(a.P, a.MZ, a.base, D, pooled);
-    if (head && pred)
-        head_kernel<<<B, 256, 0, st>>>(pooled, D, head->W, head->bias, head->centers, head->K, pred);
+    if (head && pred) {
+        const int vec4 = (D % 4 == 0) && aligned16(head->W) && aligned16(pooled);
+        head_kernel<<<B, 1024, 0, st>>>(pooled, D, head->W, head->bias, head->centers, head->K,
+                                        vec4, pred);
+    }
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "pool launch");
 }

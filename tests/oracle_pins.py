@@ -197,6 +197,23 @@ def pin_importance_gqa_and_scale():
                _brute_colsum(Q, K, cu, 0.4, heads=[h]), rtol=1e-11, what=f"head {h}")
 
 
+def pin_importance_rows_from():
+    """Forming only rows i >= r gives the exact column sums of keys j >= r (they receive
+    mass only from those rows) and strictly less for earlier keys."""
+    rng = _rng(13)
+    cu = np.asarray([0, 40, 43], dtype=np.int32)
+    Q, K = _qk(rng, cu, 4, 2, 8, spread=1.5)
+    full = oracle.attn_colsum(Q, K, cu, 0.3, exclude_self=True)
+    for r in (0, 5, 39):
+        part = oracle.attn_colsum_rows(Q, K, cu, 0.3, r, exclude_self=True)
+        for b in range(2):
+            lo, hi = cu[b], cu[b + 1]
+            late = np.arange(lo, hi) >= lo + r
+            _close(part[lo:hi][late], full[lo:hi][late], rtol=1e-12, what=f"rows_from {r}")
+            if r > 0:
+                assert np.all(part[lo:hi][~late] < full[lo:hi][~late] + 1e-15)
+
+
 def pin_lse_library():
     """Row log-normalisers equal scipy.special.logsumexp over the causal prefix."""
     rng = _rng(7)

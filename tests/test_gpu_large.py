@@ -1,0 +1,76 @@
+"""Full-size importance and pooling on the three large workloads (GPU).
+
+The GPU runs the whole workload: every prompt, every selected layer and head, in
+per-layer calls that accumulate, as a caller streaming one layer's Q/K at a time
+would.  Checks: S is finite, non-negative and sums to 1 over every prompt (any size);
+and the last keys of one prompt match the oracle exactly, because C_j needs only the
+rows i >= j.  The oracle reads the inputs of that prompt back from the device: the
+device generator writes the same bits as the host one (test_gpu_synth), and host-side
+generation of these sizes would take minutes."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import assert_importance, assert_pooled, assert_pred
+from synth import device as sd
+from synth import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _bits(t):
+    return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+@pytest.mark.parametrize("w,R", [(W.C3, 8), (W.C4, 16), (W.C5, 4)], ids=lambda x: getattr(x, "name", str(x)))
+def test_importance_full_size(cuda_lib, w, R):
+    cu = w.cu_seqlens()
+    sumT = int(cu[-1])
+    lens = np.diff(cu)
+    maxT = int(lens.max())
+    b = int(np.argmax(lens)) if w.B > 8 else w.B - 1
+    t0, t1 = int(cu[b]), int(cu[b + 1])
+    T = t1 - t0
+    ctx = cuda_lib.Context(0)
+    cu_d = sd.cu_seqlens(w)
+    C = np.zeros(T)
+    sub = np.asarray([0, T], dtype=np.int32)
+    for n, layer in enumerate(w.layers):
+        Q, K = sd.qk(w, layer)
+        ctx.attn_importance(Q, K, cu_d, maxT, accumulate=n > 0)
+        Qp = np.zeros((T, w.Hq, w.d), dtype=np.uint16)
+        Qp[T - R:] = _bits(Q[t1 - R:t1])
+        Kp = _bits(K[t0:t1])
+        oracle.attn_colsum_rows(Qp, Kp, sub, w.scale, T - R, out=C)
+        del Q, K
+    S = ctx.attn_importance_finalize(len(w.layers), sumT).cpu().numpy()
+    ctx.sync_status()
+    assert np.all(np.isfinite(S)) and np.all(S >= 0)
+    sums = np.add.reduceat(S.astype(np.float64), cu[:-1])
+    assert np.max(np.abs(sums - 1.0)) < 1e-4, sums
+    ref = oracle.importance(C, sub, len(w.layers), w.Hq)[T - R:]
+    assert_importance(S[t1 - R:t1], ref)
+
+
+@pytest.mark.parametrize("w", [W.C3, W.C5], ids=lambda w: w.name)
+def test_pool_full_size(cuda_lib, w):
+    cu = w.cu_seqlens()
+    sumT = int(cu[-1])
+    rng = np.random.default_rng(4)
+    H = rng.uniform(0, 12, sumT).astype(np.float32)
+    S = (rng.uniform(0, 2, sumT) / np.repeat(np.diff(cu), np.diff(cu))).astype(np.float32)
+    ctx = cuda_lib.Context(0)
+    Wt, bias, c = w.head_params()
+    head = cuda_lib.Head(torch.from_numpy(Wt).cuda(), torch.from_numpy(bias).cuda(),
+                         torch.from_numpy(c).cuda())
+    hid = sd.hidden(w)
+    pooled, pred = ctx.pool(hid, torch.from_numpy(H).cuda(), torch.from_numpy(S).cuda(),
+                            sd.cu_seqlens(w), w.lambda1, w.lambda2, w.alpha, head=head)
+    ctx.sync_status()
+    for b in (0, w.B - 1):
+        rows = slice(int(cu[b]), int(cu[b + 1]))
+        sub = np.asarray([0, int(cu[b + 1] - cu[b])], dtype=np.int32)
+        P = oracle.pool(_bits(hid[rows]), H[rows], S[rows], sub, w.lambda1, w.lambda2, w.alpha)
+        assert_pooled(pooled[b:b + 1].cpu().numpy(), P)
+        assert_pred(pred[b:b + 1].cpu().numpy(), oracle.length_head(P, Wt, bias, c))

@@ -24,6 +24,8 @@ MUTANTS = [
     ("Q prompt offset dropped", "((t0 + t) * c->Hq + h)", "((t) * c->Hq + h)"),
     ("self term never excluded", "if (c->exclude_self && j == i) continue;", ""),
     ("lse sign", "m + log(Z);", "m - log(Z);"),
+    ("rows_from off by one", "for (int64_t i = c->row_from; i < T; ++i) {",
+     "for (int64_t i = c->row_from + 1; i < T; ++i) {"),
     ("causal count divisor", "((double)N * (double)n_layers",
      "((double)(N - j) * (double)n_layers"),
     ("head mean dropped", "(double)n_layers * (double)n_heads)", "(double)n_layers)"),
