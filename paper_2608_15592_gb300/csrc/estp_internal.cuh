@@ -21,6 +21,7 @@ struct estp_ctx {
     int32_t imp_B = 0;
     const int32_t* imp_cu = nullptr;
     int32_t imp_n_heads = 0;
+    int tc_clusters[4] = {0, 0, 0, 0};  // resident clusters of each tcgen05 kernel (0 = unknown)
 };
 
 namespace estp {

@@ -2,20 +2,27 @@
 //
 // Both kernels recompute S = Q K^T tile by tile on the 5th-generation tensor cores
 // and never materialise the attention matrix A (Sec. 3.1).  One persistent CTA per
-// SM runs a warp-specialised pipeline:
-//   warp 0      TMA producer: the item's fixed 128-row tile, then a ring of streamed
-//               128-row tiles (128B-swizzled, one 64-column atom per TMA box)
-//   warp 1      MMA issuer: D[128 x 128] (fp32, TMEM) = fixed (M side) x streamed^T,
-//               double-buffered accumulators (2 x 128 TMEM columns)
-//   warps 2-9   epilogue: tcgen05.ld of the accumulator, exp2 and row reductions;
-//               warp w reads TMEM lanes 32*(w%4).. (its quarter), and the two warps
-//               of a quarter split the 128 columns (halves)
+// SM works on "pair items": two fixed 128-row tiles (2p and 2p+1) multiplied by the
+// same sequence of streamed 128-row tiles, so that every streamed tile feeds two MMAs.
+// (Tile loads through TMA reach only ~24-34 B/clk per SM; one 128 x 128 x 128 MMA per
+// streamed tile would need ~58.)  The CTA runs a warp-specialised pipeline:
+//   warp 0       TMA producer: the item's two fixed tiles, then a ring of streamed tiles
+//                (128B-swizzled, one 64-column atom per TMA box) and, for column sums,
+//                the lse values of each streamed query tile
+//   warp 1       MMA issuer: D_A = A x S^T and D_B = B x S^T (M = 128 each, N = 128,
+//                fp32 in TMEM), double-buffered: 2 x 2 x 128 = all 512 TMEM columns
+//   warps 2-17   epilogue: warps 2-9 read D_A, warps 10-17 D_B; warp w reads TMEM lanes
+//                32*(w%4).. (its quarter), and two warps of a quarter split the 128
+//                columns (halves); tcgen05.ld, exp2 and row reductions
 //
-// LSE mode (rows = queries): lse_i = ln sum_{j<=i} exp(scale q_i.k_j), streaming the
-//   key tiles 0..qt with a running max (flash-style online normaliser).
-// Column-sum mode (rows = keys): C_j += sum_{i>=j} 2^(scale*log2e q_i.k_j - log2e*lse_i),
-//   streaming the query tiles of the item for every selected head of the KV group, so
-//   the sum over queries stays in the thread that owns key j.
+// LSE mode (rows = queries): pair p = query tiles 2p, 2p+1 of one head, streaming the
+//   key tiles 0..2p+1 with a running max (flash-style normaliser); a tile skips the
+//   key tiles after its own query tile.
+// Column-sum mode (rows = keys): pair p = key tiles 2p, 2p+1 of one KV group,
+//   C_j += sum_{i>=j} 2^(scale*log2e q_i.k_j - log2e*lse_i), streaming the query tiles
+//   of the item's chunk for every selected head of the group, so the sum over queries
+//   stays in the thread that owns key j; a tile skips query tiles before its own key
+//   tile.
 //
 // Every mbarrier wait is bounded (about 2 s of SM clock); on expiry the CTA records
 // ESTP_ERR_TIMEOUT in the status word and drains without further waits.
@@ -28,12 +35,21 @@
 namespace estp {
 namespace {
 
-constexpr int kTile = 128;
-constexpr int kQcTc = 4;
-constexpr int kThreads = 320;          // 10 warps
-constexpr int kEpiWarp0 = 2;           // warps 2..9
+constexpr int kTile = 128;             // rows of a fixed or streamed tile
+constexpr int kPair = 2 * kTile;       // rows of the fixed pair (the plan's tile)
+constexpr int kQcPair = 2;             // pairs of query tiles per column-sum item
+constexpr int kEpiWarp0 = 2;           // warps 2..17
+constexpr int kEpiWarps = 16;          // 8 per fixed tile
+constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
 constexpr int kAccCols = 128;
+constexpr int kAccBufs = 2;            // accumulator pairs in TMEM (kAccBufs x 2 x 128 columns)
 constexpr int kSched = 4;              // depth of the item-index ring (producer -> consumers)
+// Column-sum mode: the lse values of each streamed query tile reach shared memory by
+// TMA, in a ring of their own that the epilogue releases (plain loads from the epilogue
+// queue behind the tile stream and stall it for several steps).
+constexpr int kLseSlots = 8;
+constexpr int kLseBox = kTile + 4;     // floats per copy: the tile's 128, from a 16-byte boundary
+constexpr int kLseSlotBytes = 640;     // >= kLseBox * 4, multiple of 128
 
 enum Mode { kModeLse = 0, kModeImp = 1 };
 
@@ -41,19 +57,21 @@ template <int D>
 struct Cfg {
     static constexpr int kAtoms = D / 64;
     static constexpr int kTileBytes = kTile * 128 * kAtoms;  // 128 rows x D bf16
-    static constexpr int kStages = D == 64 ? 8 : 4;
+    static constexpr int kStages = D == 64 ? 6 : 2;
     static constexpr int kKSteps = D / 16;
     // dynamic smem layout (offsets from a 1024-aligned base)
-    static constexpr int kFixOff = 0;
-    static constexpr int kRingOff = 2 * kTileBytes;
-    static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [8 warps][64] f32
-    static constexpr int kMergeOff = kNlOff + 8 * 64 * 4;             // [2][4][32] float2
-    static constexpr int kBarOff = kMergeOff + 2 * 4 * 32 * 8;
-    // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[2], drain,
-    // sched_full/empty[kSched], xfull/xempty[2][4]
-    static constexpr int kNumBars = 2 + 2 + 2 * kStages + 2 + 2 + 1 + 2 * kSched + 16;
+    static constexpr int kFixOff = 0;                               // [2 buffers][A, B]
+    static constexpr int kRingOff = 4 * kTileBytes;
+    static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][64] f32
+    static constexpr int kMergeOff = kNlOff + kEpiWarps * 64 * 4;   // [2][A, B][4][32] float2
+    static constexpr int kBarOff = kMergeOff + 2 * 2 * 4 * 32 * 8;
+    // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[kAccBufs], drain,
+    // sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
+    static constexpr int kNumBars =
+        2 + 2 + 2 * kStages + 2 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
-    static constexpr int kSmemBytes = kMiscOff + 16 + 4 * kSched + 1024;  // + alignment slack
+    static constexpr int kLseOff = (kMiscOff + 16 + 4 * kSched + 127) / 128 * 128;  // lse ring
+    static constexpr int kSmemBytes = kLseOff + kLseSlots * kLseSlotBytes + 1024;  // + alignment slack
 };
 
 struct TcArgs {
@@ -78,6 +96,14 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
         "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_1d(void* dst, const CUtensorMap* map, int x, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.1d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2}], [%3];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(smem_u32(bar))
         : "memory");
 }
 
@@ -142,9 +168,10 @@ __device__ __forceinline__ void tmem_wait_ld() {
 struct TcItem {
     int b, T;
     int64_t t0;
-    int fix_y, fix_row0;       // fixed tile: head (LSE: query head, IMP: KV head), first row
+    int fix_y, fix_row0;       // fixed pair: head (LSE: query head, IMP: KV head), first row
     int n_steps;
-    // LSE: the query head; IMP: group slot, key tile, query-tile range, chunk slot
+    // LSE: the query head and the pair's first query tile (qt0);
+    // IMP: group slot, the pair's first key tile (kt), query-tile range, chunk slot
     int h, g, kt, qt0, qt1, chunk;
 };
 
@@ -152,23 +179,28 @@ template <int MODE>
 __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
     TcItem t;
     if (MODE == kModeLse) {
-        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kTile, a.hs.n_heads);
+        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kPair, a.hs.n_heads);
         t.b = li.b; t.T = li.T; t.t0 = li.t0;
         t.h = a.hs.head_list[li.hslot];
         t.fix_y = t.h;
-        t.fix_row0 = li.qt * kTile;
-        t.qt0 = li.qt;
-        t.n_steps = li.qt + 1;  // key tiles 0..qt
-        t.g = 0; t.kt = 0; t.qt1 = li.qt + 1; t.chunk = 0;
+        const int nt = (t.T + kTile - 1) / kTile;
+        t.qt0 = 2 * li.qt;                 // query tiles qt0 (A) and qt0 + 1 (B, may be >= nt)
+        t.fix_row0 = t.qt0 * kTile;
+        t.n_steps = min(t.qt0 + 2, nt);    // key tiles 0 .. the pair's last tile
+        t.g = 0; t.kt = 0; t.qt1 = t.qt0 + 2; t.chunk = 0;
     } else {
-        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kTile, kQcTc);
+        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kPair, kQcPair);
         t.b = ii.b; t.T = ii.T; t.t0 = ii.t0;
-        t.g = ii.g; t.kt = ii.kt; t.qt0 = ii.qt0; t.qt1 = ii.qt1;
-        t.chunk = (ii.qt0 - ii.kt) / kQcTc;
+        const int nt = (t.T + kTile - 1) / kTile;
+        t.g = ii.g;
+        t.kt = 2 * ii.kt;                  // key tiles kt (A) and kt + 1 (B, may be >= nt)
+        t.qt0 = 2 * ii.qt0;
+        t.qt1 = min(nt, 2 * ii.qt1);
+        t.chunk = (ii.qt0 - ii.kt) / kQcPair;
         t.fix_y = a.hs.group[ii.g];
-        t.fix_row0 = ii.kt * kTile;
+        t.fix_row0 = t.kt * kTile;
         const int nh = a.hs.begin[ii.g + 1] - a.hs.begin[ii.g];
-        t.n_steps = nh * (ii.qt1 - ii.qt0);
+        t.n_steps = nh * (t.qt1 - t.qt0);
         t.h = 0;
     }
     return t;
@@ -196,7 +228,7 @@ __device__ __forceinline__ void step_tile(const TcArgs& a, const TcItem& t, int 
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_fix, const __grid_constant__ CUtensorMap tm_str,
-                   const TcArgs a) {
+                   const __grid_constant__ CUtensorMap tm_lse, const TcArgs a) {
     using C = Cfg<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -211,12 +243,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* ring_full = bars + 4;               // [kStages]
     uint64_t* ring_empty = bars + 4 + C::kStages; // [kStages]
     uint64_t* acc_full = bars + 4 + 2 * C::kStages;
-    uint64_t* acc_empty = acc_full + 2;
-    uint64_t* drain = acc_empty + 2;
+    uint64_t* acc_empty = acc_full + kAccBufs;
+    uint64_t* drain = acc_empty + kAccBufs;
     uint64_t* sched_full = drain + 1;             // [kSched]
     uint64_t* sched_empty = sched_full + kSched;  // [kSched]
-    uint64_t* xfull = sched_empty + kSched;       // [2][4]: half-1 partials ready
-    uint64_t* xempty = xfull + 8;                 // [2][4]: half-0 has read them
+    uint64_t* xfull = sched_empty + kSched;       // [2][A, B][4]: half-1 partials ready
+    uint64_t* xempty = xfull + 16;                // [2][A, B][4]: half-0 has read them
+    uint64_t* lse_full = xempty + 16;             // [kLseSlots]
+    uint64_t* lse_empty = lse_full + kLseSlots;   // [kLseSlots]
+    float* lse_ring = reinterpret_cast<float*>(sm + C::kLseOff);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 4);
     volatile int* sched_item = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 16);
@@ -226,8 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&fix_full[i], 1);
             mbar_init(&fix_empty[i], 1);
+        }
+        for (int i = 0; i < kAccBufs; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], 8);  // one arrival per epilogue warp
+            mbar_init(&acc_empty[i], kEpiWarps);  // one arrival per epilogue warp
         }
         for (int i = 0; i < C::kStages; ++i) {
             mbar_init(&ring_full[i], 1);
@@ -236,19 +273,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(drain, 1);
         for (int i = 0; i < kSched; ++i) {
             mbar_init(&sched_full[i], 1);
-            mbar_init(&sched_empty[i], 1 + 8);  // MMA thread + 8 epilogue warps
+            mbar_init(&sched_empty[i], 1 + kEpiWarps);  // MMA thread + epilogue warps
         }
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < 16; ++i) {
             mbar_init(&xfull[i], 1);
             mbar_init(&xempty[i], 1);
+        }
+        for (int i = 0; i < kLseSlots; ++i) {
+            mbar_init(&lse_full[i], 1);
+            mbar_init(&lse_empty[i], kEpiWarps);  // one arrival per epilogue warp
         }
         *abort_flag = 0;
         mbar_fence_init();
     }
-    if (warp == 1) {  // TMEM: 2 accumulators x 128 columns
+    if (warp == 1) {  // TMEM: kAccBufs x (A, B) x 128 columns
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
-                     "r"(2 * kAccCols));
+                     "r"(kAccBufs * 2 * kAccCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     tc_fence_before();
@@ -277,7 +318,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_fix)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_str)) : "memory");
-            long long step = 0;
+            if (MODE == kModeImp)
+                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_lse)) : "memory");
+            uint32_t step = 0;
+            int n_items = 0;
             int item = blockIdx.x;
             for (int it = 0;; ++it) {
                 if (item >= total) item = -1;
@@ -291,21 +335,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
-                mbar_expect_tx(&fix_full[fb], C::kTileBytes);
+                mbar_expect_tx(&fix_full[fb], 2 * C::kTileBytes);
 #pragma unroll
-                for (int at = 0; at < C::kAtoms; ++at)
-                    tma_load_3d(fix + fb * C::kTileBytes + at * kTile * 128, &tm_fix, at * 64, t.fix_y,
-                                (int)(t.t0 + t.fix_row0), &fix_full[fb]);
+                for (int tau = 0; tau < 2; ++tau)
+#pragma unroll
+                    for (int at = 0; at < C::kAtoms; ++at)
+                        tma_load_3d(fix + (fb * 2 + tau) * C::kTileBytes + at * kTile * 128, &tm_fix,
+                                    at * 64, t.fix_y, (int)(t.t0 + t.fix_row0) + tau * kTile,
+                                    &fix_full[fb]);
+                ++n_items;
                 bool ok = true;
                 for (int s = 0; s < t.n_steps; ++s, ++step) {
                     const int stage = (int)(step % C::kStages);
-                    const long long u = step / C::kStages;
-                    if (u >= 1 && !wait_bar(&ring_empty[stage], (uint32_t)((u - 1) & 1), abort_flag, a.status)) {
+                    const uint32_t u = step / C::kStages;
+                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
                     int y, row0, head, qt;
                     step_tile<MODE>(a, t, s, y, row0, head, qt);
+                    if (MODE == kModeImp) {  // the tile's lse values, from a 16-byte boundary
+                        const int ls = (int)(step % kLseSlots);
+                        const uint32_t lu = step / kLseSlots;
+                        if (lu >= 1 && !wait_bar(&lse_empty[ls], (lu - 1) & 1, abort_flag, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        const int64_t x = (int64_t)head * a.sumT + t.t0 + row0;
+                        mbar_expect_tx(&lse_full[ls], kLseBox * 4);
+                        tma_load_1d(lse_ring + ls * (kLseSlotBytes / 4), &tm_lse, (int)(x & ~int64_t(3)),
+                                    &lse_full[ls]);
+                    }
                     mbar_expect_tx(&ring_full[stage], C::kTileBytes);
 #pragma unroll
                     for (int at = 0; at < C::kAtoms; ++at)
@@ -315,11 +375,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 item = (int)gridDim.x + atomicAdd(&info->next, 1);
             }
+            // Every copy this thread issued has landed before the CTA can exit (on the
+            // normal path the consumers already waited for all of them).
+            for (uint32_t st = 0; st < (uint32_t)C::kStages && st < step; ++st)
+                drain_wait(&ring_full[st], ((step - 1 - st) / C::kStages) & 1, a.status);
+            if (MODE == kModeImp)
+                for (uint32_t ls = 0; ls < (uint32_t)kLseSlots && ls < step; ++ls)
+                    drain_wait(&lse_full[ls], ((step - 1 - ls) / kLseSlots) & 1, a.status);
+            for (int fb = 0; fb < 2 && fb < n_items; ++fb)
+                drain_wait(&fix_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            long long step = 0;
+            uint32_t step = 0;
             bool issued = false;
             for (int it = 0;; ++it) {
                 const int item = consume_item(it, false);
@@ -327,15 +396,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
-                const uint32_t fix_addr = smem_u32(fix + fb * C::kTileBytes);
+                const uint32_t fix_addr = smem_u32(fix + fb * 2 * C::kTileBytes);  // tile A; B follows
                 bool ok = true;
                 for (int s = 0; s < t.n_steps; ++s, ++step) {
                     const int stage = (int)(step % C::kStages);
-                    const long long u = step / C::kStages;
-                    const int ab = (int)(step & 1);
-                    const long long ua = step >> 1;
-                    if (!wait_bar(&ring_full[stage], (uint32_t)(u & 1), abort_flag, a.status) ||
-                        (ua >= 1 && !wait_bar(&acc_empty[ab], (uint32_t)((ua - 1) & 1), abort_flag, a.status))) {
+                    const uint32_t u = step / C::kStages;
+                    const int ab = (int)(step % kAccBufs);
+                    const uint32_t ua = step / kAccBufs;
+                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status) ||
+                        (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
@@ -344,8 +413,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int kk = 0; kk < C::kKSteps; ++kk) {
                         const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
-                        mma_bf16(tmem + (uint32_t)(ab * kAccCols), sw128_desc(fix_addr + off),
-                                 sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
+                        const uint64_t sdesc = sw128_desc(str_addr + off);
+#pragma unroll
+                        for (int tau = 0; tau < 2; ++tau)
+                            mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
+                                     sw128_desc(fix_addr + tau * C::kTileBytes + off), sdesc,
+                                     kk > 0 ? 1u : 0u);
                     }
                     mma_commit(&ring_empty[stage]);
                     mma_commit(&acc_full[ab]);
@@ -361,11 +434,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ------------------------------------------------------------- epilogue
+        const int e = warp - kEpiWarp0;
+        const int tau = e >> 3;                    // fixed tile: 0 = A, 1 = B
         const int q = warp & 3;                    // TMEM lane quarter
-        const int half = (warp - kEpiWarp0) >> 2;  // column half
+        const int half = (e >> 2) & 1;             // column half
         const int row = q * 32 + lane;             // accumulator row owned by this thread
-        float* nl = nl_all + (warp - kEpiWarp0) * 64;
-        long long step = 0;
+        float* nl = nl_all + e * 64;
+        uint32_t step = 0;
         bool ok = true;
         for (int it = 0; ok; ++it) {
             const int item = consume_item(it, true);
@@ -373,90 +448,121 @@ __global__ void __launch_bounds__(kThreads, 1)
             const TcItem t = make_item<MODE>(a, item);
             float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
             float m = -1e30f, ssum = 0.f;          // LSE mode
-            float pre0 = 0.f, pre1 = 0.f;
-            auto load_nl = [&](int s, float& r0, float& r1) {
+            auto do_step = [&](int s) -> bool {
                 int y, row0, head, qt;
                 step_tile<MODE>(a, t, s, y, row0, head, qt);
-                const int i0 = row0 + half * 64 + lane, i1 = i0 + 32;
-                const float* l = a.lse + (int64_t)head * a.sumT + t.t0;
-                r0 = i0 < t.T ? -l[i0] * kLog2e : -INFINITY;
-                r1 = i1 < t.T ? -l[i1] * kLog2e : -INFINITY;
-            };
-            if (MODE == kModeImp) load_nl(0, pre0, pre1);
-            for (int s = 0; s < t.n_steps && ok; ++s, ++step) {
-                int y, row0, head, qt;
-                step_tile<MODE>(a, t, s, y, row0, head, qt);
-                if (MODE == kModeImp) {
+                if (MODE == kModeImp) {  // -log2e * lse of this warp's 64 query columns
+                    const int ls = (int)(step % kLseSlots);
+                    if (!warp_wait(&lse_full[ls], (step / kLseSlots) & 1, abort_flag, a.status))
+                        return false;
+                    const int64_t x = (int64_t)head * a.sumT + t.t0 + row0;
+                    const float* lr = lse_ring + ls * (kLseSlotBytes / 4) + (int)(x & 3) + half * 64;
+                    const int i0 = row0 + half * 64 + lane, i1 = i0 + 32;
+                    const float r0 = i0 < t.T ? -lr[lane] * kLog2e : -INFINITY;
+                    const float r1 = i1 < t.T ? -lr[lane + 32] * kLog2e : -INFINITY;
                     __syncwarp();
-                    nl[lane] = pre0;
-                    nl[lane + 32] = pre1;
+                    if (lane == 0) mbar_arrive(&lse_empty[ls]);
+                    nl[lane] = r0;
+                    nl[lane + 32] = r1;
                     __syncwarp();
-                    if (s + 1 < t.n_steps) load_nl(s + 1, pre0, pre1);
                 }
-                const int ab = (int)(step & 1);
-                ok = warp_wait(&acc_full[ab], (uint32_t)((step >> 1) & 1), abort_flag, a.status);
-                if (!ok) break;
+                const int ab = (int)(step % kAccBufs);
+                if (!warp_wait(&acc_full[ab], (step / kAccBufs) & 1, abort_flag, a.status))
+                    return false;
                 tc_fence_after();
-                float v[64];
-                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * kAccCols + half * 64);
-                tmem_ld32(taddr, v);
-                tmem_ld32(taddr + 32, v + 32);
-                tmem_wait_ld();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) +
+                                       (uint32_t)((ab * 2 + tau) * kAccCols + half * 64);
                 const int col0 = half * 64;
-                if (MODE == kModeImp) {
-                    const float2 sc = make_float2(a.scale_log2, a.scale_log2);
-                    if (qt != t.kt) {
+                const float2 sc = make_float2(a.scale_log2, a.scale_log2);
+                // column-sum mode: this warp's key tile against the streamed query tile
+                const int kt = t.kt + tau;
+                const bool imp_skip = MODE == kModeImp && qt < kt;   // queries all before keys
+                const bool imp_diag = MODE == kModeImp && qt == kt;
+                // LSE mode: this warp's query tile against streamed key tile s
+                const int my_qt = t.qt0 + tau;
+                const bool lse_skip = MODE == kModeLse && s > my_qt;  // keys all after queries
+                const bool lse_diag = MODE == kModeLse && s == my_qt;
+                // two chunks of 32 columns: load, (release the accumulator), reduce
 #pragma unroll
-                        for (int c = 0; c < 64; c += 4) {
-                            const float4 n4 = *reinterpret_cast<const float4*>(nl + c);
-                            float2 x0 = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, make_float2(n4.x, n4.y));
-                            float2 x1 = __ffma2_rn(make_float2(v[c + 2], v[c + 3]), sc, make_float2(n4.z, n4.w));
-                            acc2 = __fadd2_rn(acc2, make_float2(ex2(x0.x), ex2(x0.y)));
-                            acc2 = __fadd2_rn(acc2, make_float2(ex2(x1.x), ex2(x1.y)));
+                for (int ch = 0; ch < 2; ++ch) {
+                    float v[32];
+                    tmem_ld32(taddr + ch * 32, v);
+                    tmem_wait_ld();
+                    if (ch == 1) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                    }
+                    const int cb = col0 + ch * 32;  // tile column of v[0]
+                    const float* nc = nl + ch * 32;
+                    if (MODE == kModeImp) {
+                        if (imp_skip) continue;
+                        if (!imp_diag) {
+                            float2 acc_b = make_float2(0.f, 0.f);
+#pragma unroll
+                            for (int c = 0; c < 32; c += 4) {
+                                const float4 n4 = *reinterpret_cast<const float4*>(nc + c);
+                                float2 x0 = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, make_float2(n4.x, n4.y));
+                                float2 x1 = __ffma2_rn(make_float2(v[c + 2], v[c + 3]), sc, make_float2(n4.z, n4.w));
+                                acc2 = __fadd2_rn(acc2, make_float2(ex2(x0.x), ex2(x0.y)));
+                                acc_b = __fadd2_rn(acc_b, make_float2(ex2(x1.x), ex2(x1.y)));
+                            }
+                            acc2 = __fadd2_rn(acc2, acc_b);
+                        } else {  // diagonal tile: query i = col, key j = row (local); keep i >= j
+#pragma unroll
+                            for (int c = 0; c < 32; c += 2) {
+                                const float2 n2 = *reinterpret_cast<const float2*>(nc + c);
+                                float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, n2);
+                                const int i0 = cb + c, i1 = i0 + 1;
+                                const bool k0 = a.exclude_self ? i0 > row : i0 >= row;
+                                const bool k1 = a.exclude_self ? i1 > row : i1 >= row;
+                                acc2 = __fadd2_rn(acc2, make_float2(k0 ? ex2(x.x) : 0.f, k1 ? ex2(x.y) : 0.f));
+                            }
                         }
-                    } else {  // diagonal tile: query i = col, key j = row (local); keep i >= j
+                    } else {
+                        if (lse_skip) continue;
+                        if (lse_diag) {  // diagonal tile: keys j = col after the query i = row
 #pragma unroll
-                        for (int c = 0; c < 64; c += 2) {
-                            const float2 n2 = *reinterpret_cast<const float2*>(nl + c);
-                            float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, n2);
-                            const int i0 = col0 + c, i1 = i0 + 1;
-                            const bool k0 = a.exclude_self ? i0 > row : i0 >= row;
-                            const bool k1 = a.exclude_self ? i1 > row : i1 >= row;
-                            acc2 = __fadd2_rn(acc2, make_float2(k0 ? ex2(x.x) : 0.f, k1 ? ex2(x.y) : 0.f));
+                            for (int c = 0; c < 32; ++c)
+                                if (cb + c > row) v[c] = -INFINITY;
                         }
-                    }
-                } else {
-                    const bool diag = (s == t.qt0);  // key tile == query tile
-                    float mx = -1e30f;
+                        // chunk max: four independent 3-input max chains, then a short tree
+                        float mk[4];
 #pragma unroll
-                    for (int c = 0; c < 64; ++c) {
-                        if (diag && col0 + c > row) v[c] = -INFINITY;
-                        mx = fmaxf(mx, v[c]);
-                    }
-                    const float nm = fmaxf(m, mx * a.scale_log2);
-                    ssum *= ex2(m - nm);
-                    m = nm;
-                    const float2 sc = make_float2(a.scale_log2, a.scale_log2);
-                    const float2 nm2 = make_float2(-nm, -nm);
-                    float2 s2 = make_float2(0.f, 0.f);
+                        for (int k = 0; k < 4; ++k) {
+                            const float* w8 = v + 8 * k;
+                            mk[k] = fmaxf(fmax3(fmax3(w8[0], w8[1], w8[2]), w8[3], w8[4]),
+                                          fmax3(w8[5], w8[6], w8[7]));
+                        }
+                        const float mx = fmaxf(fmax3(mk[0], mk[1], mk[2]), mk[3]);
+                        const float nm = fmaxf(m, mx * a.scale_log2);
+                        ssum *= ex2(m - nm);
+                        m = nm;
+                        const float2 nm2 = make_float2(-nm, -nm);
+                        float2 s2[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                                        make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-                    for (int c = 0; c < 64; c += 2) {
-                        float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, nm2);
-                        s2 = __fadd2_rn(s2, make_float2(ex2(x.x), ex2(x.y)));
+                        for (int c = 0; c < 32; c += 2) {
+                            float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, nm2);
+                            s2[(c >> 1) & 3] = __fadd2_rn(s2[(c >> 1) & 3], make_float2(ex2(x.x), ex2(x.y)));
+                        }
+                        const float2 s01 = __fadd2_rn(s2[0], s2[1]), s23 = __fadd2_rn(s2[2], s2[3]);
+                        const float2 st = __fadd2_rn(s01, s23);
+                        ssum += st.x + st.y;
                     }
-                    ssum += s2.x + s2.y;
                 }
-            }
+                ++step;
+                return true;
+            };
+            for (int s = 0; s < t.n_steps; ++s)
+                if (!(ok = do_step(s))) break;
             if (!ok) break;
             // merge the two column halves of each row (bounded mbarrier hand-off), then write
             const int pb = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
-            float2* mb = merge + pb * 128;
-            uint64_t* xf = &xfull[pb * 4 + q];
-            uint64_t* xe = &xempty[pb * 4 + q];
+            float2* mb = merge + (pb * 2 + tau) * 128;
+            uint64_t* xf = &xfull[(pb * 2 + tau) * 4 + q];
+            uint64_t* xe = &xempty[(pb * 2 + tau) * 4 + q];
             if (half == 1) {
                 if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status);
                 if (!ok) break;
@@ -471,14 +577,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(xe);
                 if (MODE == kModeImp) {
-                    const int j = t.fix_row0 + row;
+                    const int j = t.fix_row0 + tau * kTile + row;
                     if (j < t.T)
                         a.part[((int64_t)t.chunk * a.hs.n_groups + t.g) * a.sumT + t.t0 + j] =
                             acc2.x + acc2.y + o.x;
                 } else {
                     const float mm = fmaxf(m, o.x);
                     const float ss = ssum * ex2(m - mm) + o.y * ex2(o.x - mm);
-                    const int i = t.fix_row0 + row;
+                    const int i = t.fix_row0 + tau * kTile + row;
                     if (i < t.T) a.lse_out[(int64_t)t.h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
                 }
             }
@@ -490,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 1) {
         __syncwarp();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                     "r"(2 * kAccCols));
+                     "r"(kAccBufs * 2 * kAccCols));
     }
 }
 
@@ -523,14 +629,29 @@ estp_status make_map(CUtensorMap* m, const void* base, int heads, int d, int64_t
     return ESTP_OK;
 }
 
+// lse [Hq * sumT] fp32 as a 1-D tensor; box kLseBox (outside the array reads zero).
+estp_status make_lse_map(CUtensorMap* m, const float* lse, int64_t n) {
+    auto fn = encode_fn();
+    if (!fn) return fail(ESTP_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[1] = {(cuuint64_t)n};
+    cuuint64_t strides[1] = {0};
+    cuuint32_t box[1] = {(cuuint32_t)kLseBox};
+    cuuint32_t es[1] = {1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 1, const_cast<float*>(lse), dims, strides,
+                    box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(ESTP_ERR_CUDA, "cuTensorMapEncodeTiled (lse) failed (%d)", (int)r);
+    return ESTP_OK;
+}
+
 template <int D, int MODE>
 estp_status launch_tc(estp_ctx* ctx, const CUtensorMap& fixm, const CUtensorMap& strm,
-                      const TcArgs& a, cudaStream_t st) {
+                      const CUtensorMap& lsem, const TcArgs& a, cudaStream_t st) {
     auto kern = attn_tc_kernel<D, MODE>;
     const int smem = Cfg<D>::kSmemBytes;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "tc kernel smem attribute");
-    kern<<<ctx->num_sms, kThreads, smem, st>>>(fixm, strm, a);
+    kern<<<ctx->num_sms, kThreads, smem, st>>>(fixm, strm, lsem, a);
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "tc kernel launch");
 }
@@ -538,8 +659,8 @@ estp_status launch_tc(estp_ctx* ctx, const CUtensorMap& fixm, const CUtensorMap&
 }  // namespace
 
 bool tc_supported(estp_dtype dtype, int d) { return dtype == ESTP_BF16 && (d == 64 || d == 128); }
-int tc_tile() { return kTile; }
-int tc_qc() { return kQcTc; }
+int tc_tile() { return kPair; }
+int tc_qc() { return kQcPair; }
 
 estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, int Hkv, int d,
                           float scale, const ImpHeads& hs, const int32_t* cu, int B, int64_t sumT,
@@ -559,11 +680,13 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
     CUtensorMap mq, mk;
     if ((s = make_map(&mq, Q, Hq, d, sumT)) != ESTP_OK) return s;
     if ((s = make_map(&mk, K, Hkv, d, sumT)) != ESTP_OK) return s;
-    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kTile, 1, hs.n_heads, 1,
+    // LSE pair items: (prompt, pair of query tiles, head)
+    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kPair, 1, hs.n_heads, 1,
                                          const_cast<int32_t*>(a.base), const_cast<PlanInfo*>(a.info),
                                          ctx->status);
-    return d == 64 ? launch_tc<64, kModeLse>(ctx, mq, mk, a, st)
-                   : launch_tc<128, kModeLse>(ctx, mq, mk, a, st);
+    // (the lse map argument is unused in this mode)
+    return d == 64 ? launch_tc<64, kModeLse>(ctx, mq, mk, mq, a, st)
+                   : launch_tc<128, kModeLse>(ctx, mq, mk, mq, a, st);
 }
 
 estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const float* lse, int Hq,
@@ -579,12 +702,17 @@ estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const flo
     a.part = part;
     a.status = ctx->status;
     a.hs = hs;
-    CUtensorMap mq, mk;
+    // the lse coordinate of a TMA copy is a 32-bit element index
+    if ((int64_t)Hq * sumT + kLseBox >= ((int64_t)1 << 31))
+        return fail(ESTP_ERR_UNSUPPORTED, "Hq * sumT = %lld lse values exceed 2^31 - %d",
+                    (long long)Hq * sumT, kLseBox);
+    CUtensorMap mq, mk, ml;
     estp_status s;
     if ((s = make_map(&mq, Q, Hq, d, sumT)) != ESTP_OK) return s;
     if ((s = make_map(&mk, K, Hkv, d, sumT)) != ESTP_OK) return s;
-    return d == 64 ? launch_tc<64, kModeImp>(ctx, mk, mq, a, st)
-                   : launch_tc<128, kModeImp>(ctx, mk, mq, a, st);
+    if ((s = make_lse_map(&ml, lse, (int64_t)Hq * sumT)) != ESTP_OK) return s;
+    return d == 64 ? launch_tc<64, kModeImp>(ctx, mk, mq, ml, a, st)
+                   : launch_tc<128, kModeImp>(ctx, mk, mq, ml, a, st);
 }
 
 }  // namespace estp
