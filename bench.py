@@ -190,8 +190,8 @@ class Step:
         self.pred = torch.empty(w.B, dtype=torch.float32, device=device)
         self.ctx = estp.Context(torch.cuda.current_device())
         n_layers = len(w.layers)
-        # launches per step: entropy 2; per layer lse 2 + importance 3; finalize 1; pool 4
-        self.launches = 2 + n_layers * 5 + 1 + 4
+        # launches per step: entropy 2; per layer lse 2 + importance 3; finalize 1; pool 2
+        self.launches = 2 + n_layers * 5 + 1 + 2
 
     def run(self, ev=None):
         """One step on the current stream; ev: dict of (start, end) events per kernel."""

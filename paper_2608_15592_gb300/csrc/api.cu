@@ -111,6 +111,7 @@ void estp_destroy(estp_ctx* ctx) {
     cudaDeviceSynchronize();
     cudaFree(ctx->ws);
     cudaFree(ctx->imp_acc);
+    cudaFree(ctx->pool_done);
     cudaFree(ctx->status);
     delete ctx;
 }

@@ -21,7 +21,8 @@ struct estp_ctx {
     int32_t imp_B = 0;
     const int32_t* imp_cu = nullptr;
     int32_t imp_n_heads = 0;
-    int tc_clusters[4] = {0, 0, 0, 0};  // resident clusters of each tcgen05 kernel (0 = unknown)
+    uint32_t* pool_done = nullptr;      // per-prompt arrival counters of the pooling kernel
+    int32_t pool_done_cap = 0;
 };
 
 namespace estp {

@@ -18,11 +18,13 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
                                                          int max_seqlen, int tile, int qc,
                                                          int mult, int kind, int32_t* base,
                                                          PlanInfo* info, int* status) {
-    __shared__ int32_t sums[1024];
+    // thread t owns prompts [t*per, (t+1)*per); one read of cu, warp-shuffle scans
+    __shared__ int64_t warp_sum[32];
     __shared__ int bad;
-    const int tid = threadIdx.x;
-    if (tid == 0) bad = (cu[0] != 0 || (int64_t)cu[B] != sumT);
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    if (tid == 0) bad = 0;
     __syncthreads();
+    if (tid == 0 && (cu[0] != 0 || (int64_t)cu[B] != sumT)) bad = 1;
     const int per = (B + 1023) / 1024;
     const int b0 = min(B, tid * per), b1 = min(B, b0 + per);
     int64_t local = 0;
@@ -32,27 +34,37 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
         const int nt = (len + tile - 1) / tile;
         local += (int64_t)mult * (kind == 0 ? items_f(nt, qc) : nt);
     }
-    if (local > INT32_MAX / 2) bad = 1;
-    sums[tid] = (int32_t)(local < INT32_MAX / 2 ? local : (int64_t)(INT32_MAX / 2));
-    __syncthreads();
-    for (int off = 1; off < 1024; off <<= 1) {
-        int32_t v = tid >= off ? sums[tid - off] : 0;
-        __syncthreads();
-        sums[tid] = (int32_t)(((int64_t)sums[tid] + v) < INT32_MAX / 2 ? ((int64_t)sums[tid] + v) : (int64_t)(INT32_MAX / 2));
-        __syncthreads();
+    int64_t inc = local;  // inclusive scan within the warp
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int64_t v = __shfl_up_sync(0xffffffffu, inc, off);
+        if (lane >= off) inc += v;
     }
-    const bool ok = !bad && sums[1023] < INT32_MAX / 2;
-    int32_t run = sums[tid] - (int32_t)local;
+    if (lane == 31) warp_sum[wid] = inc;
+    __syncthreads();
+    if (wid == 0) {
+        int64_t w = warp_sum[lane];
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int64_t v = __shfl_up_sync(0xffffffffu, w, off);
+            if (lane >= off) w += v;
+        }
+        warp_sum[lane] = w;  // inclusive over warps
+    }
+    __syncthreads();
+    const int64_t total = warp_sum[31];
+    const bool ok = !bad && total < INT32_MAX / 2;  // item indices stay 32-bit
+    int64_t run = inc - local + (wid > 0 ? warp_sum[wid - 1] : 0);
     for (int b = b0; b < b1; ++b) {
-        base[b] = ok ? run : 0;
+        base[b] = ok ? (int32_t)run : 0;
         const int32_t len = cu[b + 1] - cu[b];
         const int nt = (len + tile - 1) / tile;
-        if (len >= 0) run += (int32_t)((int64_t)mult * (kind == 0 ? items_f(nt, qc) : nt));
+        if (len >= 0) run += (int64_t)mult * (kind == 0 ? items_f(nt, qc) : nt);
     }
     if (tid == 1023) {
-        base[B] = ok ? sums[1023] : 0;
+        base[B] = ok ? (int32_t)total : 0;
         info->ok = ok ? 1 : 0;
-        info->total = ok ? sums[1023] : 0;
+        info->total = ok ? (int32_t)total : 0;
         info->next = 0;
     }
     if (tid == 0 && !ok) report(status, ESTP_ERR_INVALID_ARG);
@@ -248,17 +260,29 @@ __global__ void __launch_bounds__(kSThreads) imp_simt_kernel(SimtArgs a) {
 }
 
 // acc[j] (+)= sum over chunk slots c (in order) and group slots g (in order) of part.
+// Largest b with cu[b] <= j: cu staged in shared memory when it fits (kCuStage entries).
+constexpr int kCuStage = 2048;
+
+__device__ __forceinline__ const int32_t* stage_cu(const int32_t* cu, int B, int32_t* cu_s) {
+    if (B + 1 > kCuStage) return cu;
+    for (int i = threadIdx.x; i <= B; i += blockDim.x) cu_s[i] = cu[i];
+    __syncthreads();
+    return cu_s;
+}
+
 __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const int32_t* cu,
                                   int B, int64_t sumT, int n_groups, int tile, int qc,
                                   int accumulate, float* acc) {
+    __shared__ int32_t cu_s[kCuStage];
+    const int32_t* cuv = stage_cu(cu, B, cu_s);
     const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= sumT) return;
     float v = 0.f;
     if (info->ok) {
-        const int b = upper_slot(cu, B, j);
-        const int T = cu[b + 1] - cu[b];
+        const int b = upper_slot(cuv, B, j);
+        const int T = cuv[b + 1] - cuv[b];
         const int nt = (T + tile - 1) / tile;
-        const int kt = (int)((j - cu[b]) / tile);
+        const int kt = (int)((j - cuv[b]) / tile);
         const int nch = chunks_of(nt, kt, qc);
         for (int c = 0; c < nch; ++c)
             for (int g = 0; g < n_groups; ++g) v += part[((int64_t)c * n_groups + g) * sumT + j];
@@ -268,10 +292,12 @@ __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const
 
 __global__ void imp_finalize_kernel(const float* acc, const int32_t* cu, int B, int64_t sumT,
                                     float inv_lh, float* out) {
+    __shared__ int32_t cu_s[kCuStage];
+    const int32_t* cuv = stage_cu(cu, B, cu_s);
     const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= sumT) return;
-    const int b = upper_slot(cu, B, j);
-    const float N = (float)(cu[b + 1] - cu[b]);
+    const int b = upper_slot(cuv, B, j);
+    const float N = (float)(cuv[b + 1] - cuv[b]);
     out[j] = acc[j] * inv_lh / N;
 }
 

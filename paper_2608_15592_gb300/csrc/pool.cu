@@ -1,157 +1,95 @@
 // K-POOL: mixing, tempered softmax and weighted pooling (Eqs. 2-2..2-4, Sec. 3.2),
-// then the linear length head (Eq. 3-2, Sec. 3.3).
+// then the linear length head (Eq. 3-2, Sec. 3.3).  Two launches, one pass over the
+// hidden states.
 //
-// One pass over the hidden states.  Each prompt is cut into chunks of kChunk
-// tokens; a CTA owns (chunk c, slice of D) and produces
-//   M_c = max_{i in c} w_i,  Z_c = sum_{i in c} 2^(w_i - M_c),
-//   P_c = sum_{i in c} 2^(w_i - M_c) h_i,     w_i = (lambda1 S_i + lambda2 H_i) log2(e) / alpha
-// so the prompt-wide softmax of Eq. 2-3 never needs a separate pre-pass.  The merge
-// kernel combines chunks in index order:  M = max M_c,  Z = sum 2^(M_c - M) Z_c,
-// pooled = sum 2^(M_c - M) P_c / Z  (= sum_i e_i h_i, Eq. 2-4).
+// pool_stream_kernel: the packed token axis is cut evenly over a persistent grid (one
+// wave): CTA c owns tokens [t_c, t_{c+1}) with t_c = floor(c * sumT / G).  Its range
+// splits at prompt boundaries into segments; for the segment of prompt b it writes,
+// over the segment's tokens i,
+//   M = max w_i,  Z = sum 2^(w_i - M),  P = sum 2^(w_i - M) h_i,
+//   w_i = (lambda1 S_i + lambda2 H_i) log2(e) / alpha
+// (online over windows of up to 4096 tokens, rescaling when the running max grows) to
+// slot c + b.  Slots are ordered like the tokens, so the segments of a prompt occupy
+// consecutive slots.
+//
+// pool_finish_kernel: CTA (b, column block) merges the slots of prompt b in order,
+//   M* = max M_s,  Z* = sum 2^(M_s - M*) Z_s,  pooled = sum 2^(M_s - M*) P_s / Z*
+// (= sum_i e_i h_i of Eq. 2-4; zero for a prompt without tokens), and forms the partial
+// logits of the length head over its columns; the last CTA of the prompt (an arrival
+// counter) adds the partials in column-block order and reduces the head.  The merge
+// and the head run after the stream, when their short dependent reads meet an idle
+// memory system.  No floating-point atomics: every sum runs in a fixed order.
 #include "estp_internal.cuh"
 
 namespace estp {
 namespace {
 
-constexpr int kChunk = 64;        // tokens per chunk
-constexpr int kPoolThreads = 256;
-constexpr int kMergeThreads = 256;
+constexpr int kWin = 4096;        // tokens whose weights are staged at once (one window)
+constexpr int kMaxThreads = 512;  // stream CTA: 16-byte column units of one slice
+constexpr int kBatch = 8;         // rows per load batch; two batches in flight per thread
+constexpr int kFinThreads = 256;  // finish CTA: 4 columns per thread
+constexpr int kFinCols = 4 * kFinThreads;
+constexpr int kFinBins = 16;      // head bins per pass of the finish kernel
+constexpr int kMaxSlots = 1024;   // slot factors staged per pass of the finish kernel
 
-// Exclusive prefix of ceil(len_b / kChunk) over prompts, validated.  One CTA.
-__global__ void __launch_bounds__(1024) chunk_plan_kernel(const int32_t* cu, int B, int64_t sumT,
-                                                          int32_t* base, int* status) {
-    __shared__ int32_t sums[1024];
-    __shared__ int bad;
-    const int tid = threadIdx.x;
-    if (tid == 0) bad = (cu[0] != 0 || (int64_t)cu[B] != sumT);
-    __syncthreads();
-    const int per = (B + 1023) / 1024;
-    const int b0 = min(B, tid * per), b1 = min(B, b0 + per);
-    int32_t local = 0;
-    for (int b = b0; b < b1; ++b) {
-        int32_t len = cu[b + 1] - cu[b];
-        if (len < 0) bad = 1;
-        else local += (len + kChunk - 1) / kChunk;
-    }
-    sums[tid] = local;
-    __syncthreads();
-    for (int off = 1; off < 1024; off <<= 1) {  // inclusive Hillis-Steele scan
-        int32_t v = tid >= off ? sums[tid - off] : 0;
-        __syncthreads();
-        sums[tid] += v;
-        __syncthreads();
-    }
-    int32_t run = sums[tid] - local;
-    const bool ok = !bad;
-    for (int b = b0; b < b1; ++b) {
-        base[b] = ok ? run : 0;
-        int32_t len = cu[b + 1] - cu[b];
-        run += len > 0 ? (len + kChunk - 1) / kChunk : 0;
-    }
-    if (tid == 1023) base[B] = ok ? sums[1023] : 0;
-    if (tid == 0 && !ok) report(status, ESTP_ERR_INVALID_ARG);
-}
-
-struct PoolArgs {
+struct StreamArgs {
     const char* hidden;
     int64_t ld_bytes;
     int64_t D;
     int64_t units;           // 16-byte units per row covering D
+    int64_t slice_units;     // units per column slice (grid.y)
     const float* H;
     const float* S;
     const int32_t* cu;
-    const int32_t* base;     // chunk plan [B+1]
     int B;
+    int64_t sumT;
+    int G;                   // CTAs along the token axis (grid.x)
     float w_l1, w_l2;        // lambda * log2(e) / alpha
-    float* P;                // [n_chunks, D]
-    float2* MZ;              // [n_chunks] (M_c, Z_c)
+    float* P;                // [G + B slots, D]
+    float2* MZ;              // [G + B slots] (M, Z)
+    int* valid;              // 1 when cu_seqlens passed the checks (written by CTA (0, 0))
+    int* status;
 };
 
+struct FinishArgs {
+    const float* P;
+    const float2* MZ;
+    const int* valid;
+    const int32_t* cu;
+    int B;
+    int64_t sumT;
+    int G;
+    int64_t D;
+    int n_cb;                // column blocks (grid.y)
+    int vec4;                // D % 4 == 0 and P, pooled, W 16-byte aligned: float4 access
+    float* pooled;           // [B, D]
+    uint32_t* done;          // [B] arrival counters (back to zero after the last arrival)
+    float* zpart;            // [B, n_cb, K] partial logits
+    const float* W;          // length head (NULL: pooling only)
+    const float* bias;
+    const float* centers;
+    int K;
+    float* pred;
+};
+
+// Eight bf16 (or four fp32) values of one 16-byte unit, weighted by e, added to acc.
 template <bool kBf16>
-__global__ void __launch_bounds__(kPoolThreads) pool_chunk_kernel(PoolArgs a) {
-    __shared__ float e_s[kChunk];
-    __shared__ float red[2];
-    const int c = blockIdx.x;
-    if (c >= a.base[a.B]) return;
-    const int b = upper_slot(a.base, a.B, c);
-    const int64_t i0 = a.cu[b] + (int64_t)(c - a.base[b]) * kChunk;
-    const int64_t left_tokens = a.cu[b + 1] - i0;
-    const int n = left_tokens < kChunk ? (int)left_tokens : kChunk;
-    const int tid = threadIdx.x;
-    if (tid < 32) {  // chunk weights: one warp, two tokens per lane
-        float w0 = -INFINITY, w1 = -INFINITY;
-        if (tid < n) w0 = fmaf(a.w_l1, a.S[i0 + tid], a.w_l2 * a.H[i0 + tid]);
-        if (tid + 32 < n) w1 = fmaf(a.w_l1, a.S[i0 + tid + 32], a.w_l2 * a.H[i0 + tid + 32]);
-        float mx = fmaxf(w0, w1);
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-        float e0 = tid < n ? ex2(w0 - mx) : 0.f;
-        float e1 = tid + 32 < n ? ex2(w1 - mx) : 0.f;
-        e_s[tid] = e0;
-        e_s[tid + 32] = e1;
-        float z = e0 + e1;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
-        if (tid == 0) { red[0] = mx; red[1] = z; }
+__device__ __forceinline__ void acc_unit(float* acc, const uint4& v, float e) {
+    if (kBf16) {
+        acc[0] = fmaf(e, bf16lo(v.x), acc[0]);
+        acc[1] = fmaf(e, bf16hi(v.x), acc[1]);
+        acc[2] = fmaf(e, bf16lo(v.y), acc[2]);
+        acc[3] = fmaf(e, bf16hi(v.y), acc[3]);
+        acc[4] = fmaf(e, bf16lo(v.z), acc[4]);
+        acc[5] = fmaf(e, bf16hi(v.z), acc[5]);
+        acc[6] = fmaf(e, bf16lo(v.w), acc[6]);
+        acc[7] = fmaf(e, bf16hi(v.w), acc[7]);
+    } else {
+        acc[0] = fmaf(e, __uint_as_float(v.x), acc[0]);
+        acc[1] = fmaf(e, __uint_as_float(v.y), acc[1]);
+        acc[2] = fmaf(e, __uint_as_float(v.z), acc[2]);
+        acc[3] = fmaf(e, __uint_as_float(v.w), acc[3]);
     }
-    __syncthreads();
-    const int64_t u = (int64_t)blockIdx.y * kPoolThreads + tid;
-    if (blockIdx.y == 0 && tid == 0) a.MZ[c] = make_float2(red[0], red[1]);
-    if (u >= a.units) return;
-    constexpr int kPer = kBf16 ? 8 : 4;
-    float acc[kPer];
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
-    const char* p = a.hidden + i0 * a.ld_bytes + u * 16;
-    int i = 0;
-    for (; i + 8 <= n; i += 8) {
-        uint4 v[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) v[k] = ld_stream(p + (int64_t)(i + k) * a.ld_bytes);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const float e = e_s[i + k];
-            if (kBf16) {
-                acc[0] = fmaf(e, bf16lo(v[k].x), acc[0]);
-                acc[1] = fmaf(e, bf16hi(v[k].x), acc[1]);
-                acc[2] = fmaf(e, bf16lo(v[k].y), acc[2]);
-                acc[3] = fmaf(e, bf16hi(v[k].y), acc[3]);
-                acc[4] = fmaf(e, bf16lo(v[k].z), acc[4]);
-                acc[5] = fmaf(e, bf16hi(v[k].z), acc[5]);
-                acc[6] = fmaf(e, bf16lo(v[k].w), acc[6]);
-                acc[7] = fmaf(e, bf16hi(v[k].w), acc[7]);
-            } else {
-                acc[0] = fmaf(e, __uint_as_float(v[k].x), acc[0]);
-                acc[1] = fmaf(e, __uint_as_float(v[k].y), acc[1]);
-                acc[2] = fmaf(e, __uint_as_float(v[k].z), acc[2]);
-                acc[3] = fmaf(e, __uint_as_float(v[k].w), acc[3]);
-            }
-        }
-    }
-    for (; i < n; ++i) {
-        uint4 v = ld_stream(p + (int64_t)i * a.ld_bytes);
-        const float e = e_s[i];
-        if (kBf16) {
-            acc[0] = fmaf(e, bf16lo(v.x), acc[0]);
-            acc[1] = fmaf(e, bf16hi(v.x), acc[1]);
-            acc[2] = fmaf(e, bf16lo(v.y), acc[2]);
-            acc[3] = fmaf(e, bf16hi(v.y), acc[3]);
-            acc[4] = fmaf(e, bf16lo(v.z), acc[4]);
-            acc[5] = fmaf(e, bf16hi(v.z), acc[5]);
-            acc[6] = fmaf(e, bf16lo(v.w), acc[6]);
-            acc[7] = fmaf(e, bf16hi(v.w), acc[7]);
-        } else {
-            acc[0] = fmaf(e, __uint_as_float(v.x), acc[0]);
-            acc[1] = fmaf(e, __uint_as_float(v.y), acc[1]);
-            acc[2] = fmaf(e, __uint_as_float(v.z), acc[2]);
-            acc[3] = fmaf(e, __uint_as_float(v.w), acc[3]);
-        }
-    }
-    float* out = a.P + (int64_t)c * a.D + u * kPer;
-    const int64_t left = a.D - u * kPer;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k)
-        if (k < left) out[k] = acc[k];
 }
 
 __device__ float block_reduce(float v, bool is_max, float* sh) {
@@ -166,104 +104,262 @@ __device__ float block_reduce(float v, bool is_max, float* sh) {
     __syncthreads();
     float r = sh[0];
     for (int k = 1; k < nw; ++k) r = is_max ? fmaxf(r, sh[k]) : r + sh[k];
+    __syncthreads();  // sh may be reused right away
     return r;
 }
 
-// pooled[b, cols of this CTA] from the prompt's chunks, in chunk order.
-__global__ void __launch_bounds__(kMergeThreads) pool_merge_kernel(const float* P, const float2* MZ,
-                                                                   const int32_t* base, int64_t D,
-                                                                   float* pooled) {
-    __shared__ float f_s[kMergeThreads];
+// First token of CTA c's range, and the CTA that owns token i (0 <= i < sumT).
+__device__ __forceinline__ int64_t range_start(int64_t c, int64_t sumT, int G) {
+    return c * sumT / G;
+}
+__device__ __forceinline__ int owner_cta(int64_t i, int64_t sumT, int G) {
+    const int64_t c = ((i + 1) * G - 1) / sumT;
+    return (int)(c < G - 1 ? c : G - 1);
+}
+
+template <bool kBf16>
+__global__ void __launch_bounds__(kMaxThreads, 1) pool_stream_kernel(const StreamArgs a) {
+    __shared__ float e_s[kWin];
     __shared__ float sh[32];
-    const int b = blockIdx.x;
-    const int c0 = base[b], c1 = base[b + 1];
-    const int64_t col = ((int64_t)blockIdx.y * kMergeThreads + threadIdx.x) * 4;
-    float mx = -INFINITY;
-    for (int c = c0 + threadIdx.x; c < c1; c += kMergeThreads) mx = fmaxf(mx, MZ[c].x);
-    mx = block_reduce(mx, true, sh);
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    float zpart = 0.f;
-    for (int cb = c0; cb < c1; cb += kMergeThreads) {
-        __syncthreads();
-        const int c = cb + threadIdx.x;
-        float f = 0.f;
-        if (c < c1) {
-            float2 mz = MZ[c];
-            f = ex2(mz.x - mx);
-            zpart += f * mz.y;
-        }
-        f_s[threadIdx.x] = f;
-        __syncthreads();
-        const int nb = min(kMergeThreads, c1 - cb);
-        if (col < D) {
-            for (int k = 0; k < nb; ++k) {
-                const float* row = P + (int64_t)(cb + k) * D + col;
-                const float f2 = f_s[k];
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    if (col + q < D) acc[q] = fmaf(f2, row[q], acc[q]);
-            }
-        }
+    const int c = blockIdx.x, tid = threadIdx.x;
+    const int64_t t_lo = range_start(c, a.sumT, a.G), t_hi = range_start(c + 1, a.sumT, a.G);
+    const int64_t u = (int64_t)blockIdx.y * a.slice_units + tid;
+    const bool active = tid < a.slice_units && u < a.units;
+    constexpr int kPer = kBf16 ? 8 : 4;
+
+    // Every CTA checks all of cu_seqlens the same way (bad metadata: nothing is written
+    // but the flag and the status word).
+    int bad = 0;
+    if (tid == 0) bad = a.cu[0] != 0 || (int64_t)a.cu[a.B] != a.sumT;
+    for (int b = tid; b < a.B; b += blockDim.x) bad |= a.cu[b + 1] < a.cu[b];
+    bad = __syncthreads_or(bad);
+    // the finish kernel may be scheduled now: it waits for this grid before reading its output
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (c == 0 && blockIdx.y == 0 && tid == 0) {
+        *a.valid = bad ? 0 : 1;
+        if (bad) report(a.status, ESTP_ERR_INVALID_ARG);
     }
-    const float Z = block_reduce(zpart, false, sh);
-    if (col < D) {
-        const float inv = c1 > c0 ? 1.f / Z : 0.f;
+    if (bad || t_lo >= t_hi) return;
+
+    const char* p = a.hidden + (active ? u : 0) * 16;
+    int b = upper_slot(a.cu, a.B, t_lo);  // the prompt of token t_lo (never an empty one)
+    for (int64_t s0 = t_lo; s0 < t_hi;) {
+        const int64_t s1 = min((int64_t)a.cu[b + 1], t_hi);  // segment [s0, s1) of prompt b
+        float acc[kPer];
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-            if (col + q < D) pooled[(int64_t)b * D + col + q] = acc[q] * inv;
+        for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
+        float m = -INFINITY, z = 0.f;  // running max and sum (uniform over the CTA)
+        for (int64_t i0 = s0; i0 < s1; i0 += kWin) {
+            const int n = (int)min((int64_t)kWin, s1 - i0);
+            uint4 va[kBatch], vb[kBatch];  // the first rows are requested before the weights
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k)
+                if (active && k < n) va[k] = ld_stream(p + (i0 + k) * a.ld_bytes);
+            // the window's weights, its max, and 2^(w - max) staged in shared memory
+            float wmax = -INFINITY;
+            for (int i = tid; i < n; i += blockDim.x) {
+                const float w = fmaf(a.w_l1, a.S[i0 + i], a.w_l2 * a.H[i0 + i]);
+                e_s[i] = w;
+                wmax = fmaxf(wmax, w);
+            }
+            const float nm = fmaxf(m, block_reduce(wmax, true, sh));
+            float zw = 0.f;
+            for (int i = tid; i < n; i += blockDim.x) {
+                const float e = ex2(e_s[i] - nm);
+                e_s[i] = e;
+                zw += e;
+            }
+            zw = block_reduce(zw, false, sh);  // fixed-order sum (also a barrier for e_s)
+            const float f = m == -INFINITY ? 0.f : ex2(m - nm);  // rescale to the new max
+#pragma unroll
+            for (int k = 0; k < kPer; ++k) acc[k] *= f;
+            z = z * f + zw;
+            m = nm;
+            if (active) {  // rows in two alternating batches: one reduced while one loads
+                for (int i = 0; i < n; i += 2 * kBatch) {
+#pragma unroll
+                    for (int k = 0; k < kBatch; ++k)
+                        if (i + kBatch + k < n) vb[k] = ld_stream(p + (i0 + i + kBatch + k) * a.ld_bytes);
+#pragma unroll
+                    for (int k = 0; k < kBatch; ++k)
+                        if (i + k < n) acc_unit<kBf16>(acc, va[k], e_s[i + k]);
+#pragma unroll
+                    for (int k = 0; k < kBatch; ++k)
+                        if (i + 2 * kBatch + k < n) va[k] = ld_stream(p + (i0 + i + 2 * kBatch + k) * a.ld_bytes);
+#pragma unroll
+                    for (int k = 0; k < kBatch; ++k)
+                        if (i + kBatch + k < n) acc_unit<kBf16>(acc, vb[k], e_s[i + kBatch + k]);
+                }
+            }
+            __syncthreads();  // e_s is rewritten by the next window
+        }
+        const int slot = c + b;
+        if (active) {
+            float* out = a.P + (int64_t)slot * a.D + u * kPer;
+            const int64_t left = a.D - u * kPer;
+#pragma unroll
+            for (int k = 0; k < kPer; ++k)
+                if (k < left) out[k] = acc[k];
+        }
+        if (blockIdx.y == 0 && tid == 0) a.MZ[slot] = make_float2(m, z);
+        s0 = s1;
+        ++b;
+        while (b < a.B && a.cu[b + 1] == a.cu[b]) ++b;  // empty prompts own no tokens
     }
 }
 
-// Linear head + softmax over K bins + expectation (Eq. 3-2).  One CTA of 32 warps per
-// prompt; warp w forms the logits z_k = W_k . h + bias_k of bins k = w, w + 32, ...
-// (float4 loads when rows are 16-byte aligned), then the CTA reduces the softmax and
-// the expectation in a fixed order.
-__global__ void __launch_bounds__(1024) head_kernel(const float* pooled, int64_t D, const float* W,
-                                                    const float* bias, const float* centers, int K,
-                                                    int vec4, float* pred) {
+// Online merge of (max, sum) pairs: (m, z) <- (m, z) + (m2, z2) rescaled to the larger max.
+__device__ __forceinline__ void merge_mz(float& m, float& z, float m2, float z2) {
+    const float nm = fmaxf(m, m2);
+    if (nm == -INFINITY) return;
+    z = z * ex2(m - nm) + z2 * ex2(m2 - nm);
+    m = nm;
+}
+
+// 4 columns at `col` of a float row (float4 when aligned, else bounds-checked scalars).
+__device__ __forceinline__ float4 load4(const float* row, int64_t col, int64_t D, bool v4) {
+    if (v4) return *reinterpret_cast<const float4*>(row + col);
+    return make_float4(row[col], col + 1 < D ? row[col + 1] : 0.f, col + 2 < D ? row[col + 2] : 0.f,
+                       col + 3 < D ? row[col + 3] : 0.f);
+}
+
+__device__ __forceinline__ void fma4(float4& acc, float f, const float4& p) {
+    acc.x = fmaf(f, p.x, acc.x);
+    acc.y = fmaf(f, p.y, acc.y);
+    acc.z = fmaf(f, p.z, acc.z);
+    acc.w = fmaf(f, p.w, acc.w);
+}
+
+// CTA (b, column block): merge of prompt b's slots over 1024 columns, partial logits.
+__global__ void __launch_bounds__(kFinThreads) pool_finish_kernel(const FinishArgs a) {
+    __shared__ float f_s[kMaxSlots];
+    __shared__ float2 mz_s[kFinThreads / 32];
+    __shared__ float red[kFinThreads / 32][kFinBins];
     __shared__ float z_s[1024];
     __shared__ float sh[32];
-    const int b = blockIdx.x;
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    const float* h = pooled + (int64_t)b * D;
-    for (int k = wid; k < K; k += 32) {
-        const float* w = W + (int64_t)k * D;
-        float acc0 = 0.f, acc1 = 0.f;
-        if (vec4) {
-            const float4* w4 = reinterpret_cast<const float4*>(w);
-            const float4* h4 = reinterpret_cast<const float4*>(h);
-            const int64_t n4 = D / 4;
-            int64_t x = lane;
-            for (; x + 32 < n4; x += 64) {
-                const float4 a0 = w4[x], b0 = h4[x], a1 = w4[x + 32], b1 = h4[x + 32];
-                acc0 = fmaf(a0.x, b0.x, fmaf(a0.y, b0.y, fmaf(a0.z, b0.z, fmaf(a0.w, b0.w, acc0))));
-                acc1 = fmaf(a1.x, b1.x, fmaf(a1.y, b1.y, fmaf(a1.z, b1.z, fmaf(a1.w, b1.w, acc1))));
-            }
-            for (; x < n4; x += 32) {
-                const float4 a0 = w4[x], b0 = h4[x];
-                acc0 = fmaf(a0.x, b0.x, fmaf(a0.y, b0.y, fmaf(a0.z, b0.z, fmaf(a0.w, b0.w, acc0))));
-            }
-        } else {
-            for (int64_t x = lane; x < D; x += 32) acc0 = fmaf(w[x], h[x], acc0);
-        }
-        float acc = acc0 + acc1;
+    __shared__ int last;
+    const int b = blockIdx.x, cb = blockIdx.y, tid = threadIdx.x;
+    const int lane = tid & 31, wid = tid >> 5, nw = blockDim.x >> 5;
+    const int64_t col = (int64_t)cb * kFinCols + 4 * tid;  // this thread's 4 columns
+    const bool in = col < a.D;
+    const bool v4 = a.vec4 != 0;
+    // head rows of the first kFinBins bins: requested before the merge, which they do
+    // not depend on
+    float4 wv[kFinBins];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-        if (lane == 0) z_s[k] = acc + (bias ? bias[k] : 0.f);
+    for (int j = 0; j < kFinBins; ++j)
+        wv[j] = a.W && j < a.K && in ? load4(a.W + (int64_t)j * a.D, col, a.D, v4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    // the stream kernel's slots (and its verdict on cu_seqlens) are complete past this point
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (!*a.valid) return;
+    const int32_t t0 = a.cu[b], t1 = a.cu[b + 1];
+    float4 h = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (t1 > t0) {
+        const int c0 = owner_cta(t0, a.sumT, a.G), c1 = owner_cta(t1 - 1, a.sumT, a.G);
+        const int n = c1 - c0 + 1;
+        // (M*, Z*) in one pass: online per thread, then warps and the CTA in fixed order
+        float m = -INFINITY, z = 0.f;
+        for (int k = tid; k < n; k += blockDim.x) {
+            const float2 mz = a.MZ[c0 + k + b];
+            if (k < kMaxSlots) f_s[k] = mz.x;
+            merge_mz(m, z, mz.x, mz.y);
+        }
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, m, off), z2 = __shfl_xor_sync(0xffffffffu, z, off);
+            merge_mz(m, z, m2, z2);
+        }
+        if (lane == 0) mz_s[wid] = make_float2(m, z);
+        __syncthreads();
+        m = -INFINITY;
+        z = 0.f;
+        for (int w = 0; w < nw; ++w) merge_mz(m, z, mz_s[w].x, mz_s[w].y);
+        const float mx = m, inv = 1.f / z;
+        for (int cc = 0; cc < n; cc += kMaxSlots) {  // slots in passes of kMaxSlots factors
+            const int nn = min(kMaxSlots, n - cc);
+            if (cc > 0) {
+                __syncthreads();
+                for (int k = tid; k < nn; k += blockDim.x) f_s[k] = a.MZ[c0 + cc + k + b].x;
+            }
+            __syncthreads();
+            for (int k = tid; k < nn; k += blockDim.x) f_s[k] = ex2(f_s[k] - mx);
+            __syncthreads();
+            if (in) {
+                int k = 0;
+                for (; k + 8 <= nn; k += 8) {  // eight slots in flight
+                    float4 p[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) p[j] = load4(a.P + (int64_t)(c0 + cc + k + j + b) * a.D, col, a.D, v4);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) fma4(h, f_s[k + j], p[j]);
+                }
+                for (; k < nn; ++k) fma4(h, f_s[k], load4(a.P + (int64_t)(c0 + cc + k + b) * a.D, col, a.D, v4));
+            }
+        }
+        h.x *= inv; h.y *= inv; h.z *= inv; h.w *= inv;
+    }
+    if (in) {
+        float* out = a.pooled + (int64_t)b * a.D;
+        if (v4) *reinterpret_cast<float4*>(out + col) = h;
+        else {
+            out[col] = h.x;
+            if (col + 1 < a.D) out[col + 1] = h.y;
+            if (col + 2 < a.D) out[col + 2] = h.z;
+            if (col + 3 < a.D) out[col + 3] = h.w;
+        }
+    }
+    if (!a.W) return;
+    // partial logits of these columns, kFinBins bins per pass; warp partials in warp order
+    for (int k0 = 0; k0 < a.K; k0 += kFinBins) {
+        float part[kFinBins];
+#pragma unroll
+        for (int j = 0; j < kFinBins; ++j) {
+            if (k0 > 0)
+                wv[j] = k0 + j < a.K && in ? load4(a.W + (int64_t)(k0 + j) * a.D, col, a.D, v4)
+                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int j = 0; j < kFinBins; ++j) {
+            part[j] = fmaf(wv[j].x, h.x, fmaf(wv[j].y, h.y, fmaf(wv[j].z, h.z, wv[j].w * h.w)));
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) part[j] += __shfl_xor_sync(0xffffffffu, part[j], off);
+        }
+        if (lane == 0)
+#pragma unroll
+            for (int j = 0; j < kFinBins; ++j) red[wid][j] = part[j];
+        __syncthreads();
+        if (tid < kFinBins && k0 + tid < a.K) {
+            float zk = 0.f;
+            for (int w = 0; w < nw; ++w) zk += red[w][tid];
+            a.zpart[((int64_t)b * a.n_cb + cb) * a.K + k0 + tid] = zk;
+        }
+        __syncthreads();
+    }
+    // arrival; the last CTA of prompt b adds the column blocks in order and reduces the head
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) last = atomicInc(&a.done[b], (uint32_t)a.n_cb - 1) == (uint32_t)a.n_cb - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    for (int k = tid; k < a.K; k += blockDim.x) {
+        float zk = a.bias ? a.bias[k] : 0.f;
+        for (int j = 0; j < a.n_cb; ++j) zk += __ldcg(a.zpart + ((int64_t)b * a.n_cb + j) * a.K + k);
+        z_s[k] = zk;
     }
     __syncthreads();
     float mx = -INFINITY;
-    for (int k = threadIdx.x; k < K; k += 1024) mx = fmaxf(mx, z_s[k]);
+    for (int k = tid; k < a.K; k += blockDim.x) mx = fmaxf(mx, z_s[k]);
     mx = block_reduce(mx, true, sh);
     float zs = 0.f, ys = 0.f;
-    for (int k = threadIdx.x; k < K; k += 1024) {
+    for (int k = tid; k < a.K; k += blockDim.x) {
         const float e = ex2((z_s[k] - mx) * kLog2e);
         zs += e;
-        ys = fmaf(e, centers[k], ys);
+        ys = fmaf(e, a.centers[k], ys);
     }
     zs = block_reduce(zs, false, sh);
     ys = block_reduce(ys, false, sh);
-    if (threadIdx.x == 0) pred[b] = ys / zs;
+    if (tid == 0) a.pred[b] = ys / zs;
 }
 
 }  // namespace
@@ -272,43 +368,97 @@ estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int
                         int64_t ldh, const float* H, const float* S, const int32_t* cu, int B,
                         int64_t sumT, estp_mix_params mix, const estp_head* head, float* pooled,
                         float* pred, cudaStream_t st) {
-    const int64_t n_chunks = (sumT + kChunk - 1) / kChunk + B;  // upper bound
-    const size_t off_base = 0;
-    const size_t off_mz = align_up(sizeof(int32_t) * (size_t)(B + 1), 256);
-    const size_t off_p = align_up(off_mz + sizeof(float2) * (size_t)n_chunks, 256);
-    const size_t bytes = off_p + sizeof(float) * (size_t)n_chunks * (size_t)D;
-    estp_status s = ws_reserve(ctx, bytes);
-    if (s != ESTP_OK) return s;
-    char* ws = static_cast<char*>(ctx->ws);
-    PoolArgs a;
+    StreamArgs a{};
     a.hidden = static_cast<const char*>(hidden);
     a.ld_bytes = ldh * esize(dtype);
     a.D = D;
     const int per = dtype == ESTP_BF16 ? 8 : 4;
     a.units = (D + per - 1) / per;
+    const int n_slices = (int)((a.units + kMaxThreads - 1) / kMaxThreads);
+    a.slice_units = (a.units + n_slices - 1) / n_slices;
+    const int threads = (int)((a.slice_units + 31) / 32 * 32);
+    const void* kfn = dtype == ESTP_BF16 ? (const void*)pool_stream_kernel<true>
+                                         : (const void*)pool_stream_kernel<false>;
+    int occ = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kfn, threads, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "pool occupancy");
+    // one wave: G token ranges x n_slices column slices; every range holds >= 1 token
+    int64_t G = (int64_t)ctx->num_sms * (occ > 0 ? occ : 1) / n_slices;
+    if (G < 1) G = 1;
+    if (sumT > 0 && G > sumT) G = sumT;
+    a.G = (int)G;
     a.H = H;
     a.S = S;
     a.cu = cu;
-    a.base = reinterpret_cast<int32_t*>(ws + off_base);
     a.B = B;
+    a.sumT = sumT;
     a.w_l1 = mix.lambda1 * kLog2e / mix.alpha;
     a.w_l2 = mix.lambda2 * kLog2e / mix.alpha;
-    a.P = reinterpret_cast<float*>(ws + off_p);
+    a.status = ctx->status;
+    const bool with_head = head && pred;
+    const int K = with_head ? head->K : 0;
+    const int n_cb = (int)((D + kFinCols - 1) / kFinCols);
+    // arrival counters persist in the context (zero, and back to zero after each prompt)
+    if (with_head && ctx->pool_done_cap < B) {
+        cudaFree(ctx->pool_done);
+        ctx->pool_done = nullptr;
+        ctx->pool_done_cap = 0;
+        e = cudaMalloc(&ctx->pool_done, sizeof(uint32_t) * (size_t)B);
+        if (e == cudaSuccess) e = cudaMemset(ctx->pool_done, 0, sizeof(uint32_t) * (size_t)B);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(ESTP_ERR_WORKSPACE, "pool counters: %s", cudaGetErrorString(e));
+        }
+        ctx->pool_done_cap = B;
+    }
+    // workspace: [valid][MZ slots][zpart B x n_cb x K][P slots x D], G + B slots
+    const int64_t slots = G + B;
+    const size_t off_mz = 256;
+    const size_t off_z = align_up(off_mz + sizeof(float2) * (size_t)slots, 256);
+    const size_t off_p = align_up(off_z + sizeof(float) * (size_t)B * n_cb * K, 256);
+    estp_status s = ws_reserve(ctx, off_p + sizeof(float) * (size_t)slots * (size_t)D);
+    if (s != ESTP_OK) return s;
+    char* ws = static_cast<char*>(ctx->ws);
+    a.valid = reinterpret_cast<int*>(ws);
     a.MZ = reinterpret_cast<float2*>(ws + off_mz);
-    chunk_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, reinterpret_cast<int32_t*>(ws + off_base), ctx->status);
-    if (n_chunks > 0 && sumT > 0) {
-        dim3 grid((unsigned)n_chunks, (unsigned)((a.units + kPoolThreads - 1) / kPoolThreads));
-        if (dtype == ESTP_BF16) pool_chunk_kernel<true><<<grid, kPoolThreads, 0, st>>>(a);
-        else pool_chunk_kernel<false><<<grid, kPoolThreads, 0, st>>>(a);
+    a.P = reinterpret_cast<float*>(ws + off_p);
+    dim3 grid((unsigned)G, (unsigned)n_slices);
+    if (dtype == ESTP_BF16) pool_stream_kernel<true><<<grid, threads, 0, st>>>(a);
+    else pool_stream_kernel<false><<<grid, threads, 0, st>>>(a);
+    FinishArgs f{};
+    f.P = a.P;
+    f.MZ = a.MZ;
+    f.valid = a.valid;
+    f.cu = cu;
+    f.B = B;
+    f.sumT = sumT;
+    f.G = a.G;
+    f.D = D;
+    f.n_cb = n_cb;
+    f.vec4 = D % 4 == 0 && aligned16(pooled) && (!with_head || aligned16(head->W));
+    f.pooled = pooled;
+    if (with_head) {
+        f.done = ctx->pool_done;
+        f.zpart = reinterpret_cast<float*>(ws + off_z);
+        f.W = head->W;
+        f.bias = head->bias;
+        f.centers = head->centers;
+        f.K = K;
+        f.pred = pred;
     }
-    dim3 mgrid((unsigned)B, (unsigned)((D + 4 * kMergeThreads - 1) / (4 * kMergeThreads)));
-    pool_merge_kernel<<<mgrid, kMergeThreads, 0, st>>>(a.P, a.MZ, a.base, D, pooled);
-    if (head && pred) {
-        const int vec4 = (D % 4 == 0) && aligned16(head->W) && aligned16(pooled);
-        head_kernel<<<B, 1024, 0, st>>>(pooled, D, head->W, head->bias, head->centers, head->K,
-                                        vec4, pred);
-    }
-    cudaError_t e = cudaGetLastError();
+    // launched as a programmatic dependent of the stream kernel (it waits on it on the device)
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)B, (unsigned)n_cb);
+    cfg.blockDim = dim3(kFinThreads);
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, pool_finish_kernel, f);
+    if (e != cudaSuccess) return cuda_fail(e, "pool finish launch");
+    e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "pool launch");
 }
 

@@ -96,3 +96,20 @@ def test_pool_workload(cuda_lib, w):
                         w.alpha)
         assert_pooled(pooled[bb:bb + 1].cpu().numpy(), P)
         assert_pred(pred[bb:bb + 1].cpu().numpy(), oracle.length_head(P, Wt, b, c))
+
+
+@pytest.mark.parametrize("K,with_bias", [(1, True), (7, False), (1024, True)])
+def test_head_bins(cuda_lib, K, with_bias):
+    """Length head at the bin-count limits, with and without a bias (Eq. 3-2)."""
+    cu, hid, H, S, hd = _inputs(synth.BF16, [300, 0, 77, 1500], 3584)
+    Wt, b, c = _head(K, 3584, seed=K)
+    ctx = cuda_lib.Context(0)
+    head = cuda_lib.Head(torch.from_numpy(Wt).cuda(),
+                         torch.from_numpy(b).cuda() if with_bias else None,
+                         torch.from_numpy(c).cuda())
+    pooled, pred = ctx.pool(hd, torch.from_numpy(H).cuda(), torch.from_numpy(S).cuda(),
+                            torch.as_tensor(cu, device="cuda"), 0.7, 0.3, 1.0, head=head)
+    ctx.sync_status()
+    P_ref = oracle.pool(hid, H.astype(np.float64), S.astype(np.float64), cu, 0.7, 0.3, 1.0)
+    assert_pooled(pooled.cpu().numpy(), P_ref)
+    assert_pred(pred.cpu().numpy(), oracle.length_head(P_ref, Wt, b if with_bias else None, c))
