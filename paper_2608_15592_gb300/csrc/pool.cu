@@ -26,10 +26,9 @@ namespace {
 
 constexpr int kWin = 4096;        // tokens whose weights are staged at once (one window)
 constexpr int kMaxThreads = 512;  // stream CTA: 16-byte column units of one slice
-constexpr int kBatch = 8;         // rows per load batch; two batches in flight per thread
-constexpr int kFinThreads = 256;  // finish CTA: 4 columns per thread
-constexpr int kFinCols = 4 * kFinThreads;
-constexpr int kFinBins = 16;      // head bins per pass of the finish kernel
+constexpr int kBatch = 4;         // rows per load batch; two batches in flight per thread
+constexpr int kFinThreads = 512;  // finish CTA: 2 columns per thread
+constexpr int kFinCols = 2 * kFinThreads;
 constexpr int kMaxSlots = 1024;   // slot factors staged per pass of the finish kernel
 
 struct StreamArgs {
@@ -47,21 +46,19 @@ struct StreamArgs {
     float w_l1, w_l2;        // lambda * log2(e) / alpha
     float* P;                // [G + B slots, D]
     float2* MZ;              // [G + B slots] (M, Z)
-    int* valid;              // 1 when cu_seqlens passed the checks (written by CTA (0, 0))
     int* status;
 };
 
 struct FinishArgs {
     const float* P;
     const float2* MZ;
-    const int* valid;
     const int32_t* cu;
     int B;
     int64_t sumT;
     int G;
     int64_t D;
     int n_cb;                // column blocks (grid.y)
-    int vec4;                // D % 4 == 0 and P, pooled, W 16-byte aligned: float4 access
+    int vec2;                // D even and P, pooled, W 8-byte aligned: float2 access
     float* pooled;           // [B, D]
     uint32_t* done;          // [B] arrival counters (back to zero after the last arrival)
     float* zpart;            // [B, n_cb, K] partial logits
@@ -118,7 +115,7 @@ __device__ __forceinline__ int owner_cta(int64_t i, int64_t sumT, int G) {
 }
 
 template <bool kBf16>
-__global__ void __launch_bounds__(kMaxThreads, 1) pool_stream_kernel(const StreamArgs a) {
+__global__ void __launch_bounds__(kMaxThreads, 2) pool_stream_kernel(const StreamArgs a) {
     __shared__ float e_s[kWin];
     __shared__ float sh[32];
     const int c = blockIdx.x, tid = threadIdx.x;
@@ -128,17 +125,14 @@ __global__ void __launch_bounds__(kMaxThreads, 1) pool_stream_kernel(const Strea
     constexpr int kPer = kBf16 ? 8 : 4;
 
     // Every CTA checks all of cu_seqlens the same way (bad metadata: nothing is written
-    // but the flag and the status word).
+    // but the status word).
     int bad = 0;
     if (tid == 0) bad = a.cu[0] != 0 || (int64_t)a.cu[a.B] != a.sumT;
     for (int b = tid; b < a.B; b += blockDim.x) bad |= a.cu[b + 1] < a.cu[b];
     bad = __syncthreads_or(bad);
     // the finish kernel may be scheduled now: it waits for this grid before reading its output
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    if (c == 0 && blockIdx.y == 0 && tid == 0) {
-        *a.valid = bad ? 0 : 1;
-        if (bad) report(a.status, ESTP_ERR_INVALID_ARG);
-    }
+    if (bad && c == 0 && blockIdx.y == 0 && tid == 0) report(a.status, ESTP_ERR_INVALID_ARG);
     if (bad || t_lo >= t_hi) return;
 
     const char* p = a.hidden + (active ? u : 0) * 16;
@@ -216,44 +210,57 @@ __device__ __forceinline__ void merge_mz(float& m, float& z, float m2, float z2)
     m = nm;
 }
 
-// 4 columns at `col` of a float row (float4 when aligned, else bounds-checked scalars).
-__device__ __forceinline__ float4 load4(const float* row, int64_t col, int64_t D, bool v4) {
-    if (v4) return *reinterpret_cast<const float4*>(row + col);
-    return make_float4(row[col], col + 1 < D ? row[col + 1] : 0.f, col + 2 < D ? row[col + 2] : 0.f,
-                       col + 3 < D ? row[col + 3] : 0.f);
+// 2 columns at `col` of a float row (float2 when aligned, else bounds-checked scalars).
+__device__ __forceinline__ float2 load2(const float* row, int64_t col, int64_t D, bool v2) {
+    if (v2) return *reinterpret_cast<const float2*>(row + col);
+    return make_float2(row[col], col + 1 < D ? row[col + 1] : 0.f);
 }
 
-__device__ __forceinline__ void fma4(float4& acc, float f, const float4& p) {
-    acc.x = fmaf(f, p.x, acc.x);
-    acc.y = fmaf(f, p.y, acc.y);
-    acc.z = fmaf(f, p.z, acc.z);
-    acc.w = fmaf(f, p.w, acc.w);
+// Reduce-scatter over a warp: on entry lane l holds v[0..31] (32 bins), on exit it holds
+// in v[0] the warp sum of bin l.  Five butterfly rounds of halving width; every lane
+// adds in the same order, so the result is deterministic.
+__device__ __forceinline__ float warp_reduce_scatter32(float* v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int w = 16; w >= 1; w >>= 1) {
+        const bool upper = (lane & w) != 0;  // keep bins [w, 2w) of the current block, else [0, w)
+#pragma unroll
+        for (int j = 0; j < w; ++j) {
+            const float send = upper ? v[j] : v[j + w];
+            const float keep = upper ? v[j + w] : v[j];
+            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+        }
+    }
+    return v[0];
 }
 
-// CTA (b, column block): merge of prompt b's slots over 1024 columns, partial logits.
+// CTA (b, column block): merge of prompt b's slots over kFinCols columns, partial logits.
 __global__ void __launch_bounds__(kFinThreads) pool_finish_kernel(const FinishArgs a) {
     __shared__ float f_s[kMaxSlots];
     __shared__ float2 mz_s[kFinThreads / 32];
-    __shared__ float red[kFinThreads / 32][kFinBins];
+    __shared__ float red[kFinThreads / 32][32];
     __shared__ float z_s[1024];
     __shared__ float sh[32];
     __shared__ int last;
     const int b = blockIdx.x, cb = blockIdx.y, tid = threadIdx.x;
     const int lane = tid & 31, wid = tid >> 5, nw = blockDim.x >> 5;
-    const int64_t col = (int64_t)cb * kFinCols + 4 * tid;  // this thread's 4 columns
+    const int64_t col = (int64_t)cb * kFinCols + 2 * tid;  // this thread's 2 columns
     const bool in = col < a.D;
-    const bool v4 = a.vec4 != 0;
-    // head rows of the first kFinBins bins: requested before the merge, which they do
-    // not depend on
-    float4 wv[kFinBins];
+    const bool v2 = a.vec2 != 0;
+    // head rows of the first 32 bins: requested before the stream kernel has finished
+    float2 wv[32];
 #pragma unroll
-    for (int j = 0; j < kFinBins; ++j)
-        wv[j] = a.W && j < a.K && in ? load4(a.W + (int64_t)j * a.D, col, a.D, v4) : make_float4(0.f, 0.f, 0.f, 0.f);
-    // the stream kernel's slots (and its verdict on cu_seqlens) are complete past this point
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    if (!*a.valid) return;
+    for (int j = 0; j < 32; ++j)
+        wv[j] = a.W && j < a.K && in ? load2(a.W + (int64_t)j * a.D, col, a.D, v2) : make_float2(0.f, 0.f);
+    // cu_seqlens is an input: checked here as the stream kernel checks it (which reports)
     const int32_t t0 = a.cu[b], t1 = a.cu[b + 1];
-    float4 h = make_float4(0.f, 0.f, 0.f, 0.f);
+    int bad = 0;
+    if (tid == 0) bad = a.cu[0] != 0 || (int64_t)a.cu[a.B] != a.sumT;
+    for (int k = tid; k < a.B; k += blockDim.x) bad |= a.cu[k + 1] < a.cu[k];
+    if (__syncthreads_or(bad)) return;
+    // the stream kernel's slots are complete past this point
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    float2 h = make_float2(0.f, 0.f);
     if (t1 > t0) {
         const int c0 = owner_cta(t0, a.sumT, a.G), c1 = owner_cta(t1 - 1, a.sumT, a.G);
         const int n = c1 - c0 + 1;
@@ -286,49 +293,49 @@ __global__ void __launch_bounds__(kFinThreads) pool_finish_kernel(const FinishAr
             __syncthreads();
             if (in) {
                 int k = 0;
-                for (; k + 8 <= nn; k += 8) {  // eight slots in flight
-                    float4 p[8];
+                for (; k + 16 <= nn; k += 16) {  // sixteen slots in flight
+                    float2 p[16];
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) p[j] = load4(a.P + (int64_t)(c0 + cc + k + j + b) * a.D, col, a.D, v4);
+                    for (int j = 0; j < 16; ++j) p[j] = load2(a.P + (int64_t)(c0 + cc + k + j + b) * a.D, col, a.D, v2);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) fma4(h, f_s[k + j], p[j]);
+                    for (int j = 0; j < 16; ++j) {
+                        h.x = fmaf(f_s[k + j], p[j].x, h.x);
+                        h.y = fmaf(f_s[k + j], p[j].y, h.y);
+                    }
                 }
-                for (; k < nn; ++k) fma4(h, f_s[k], load4(a.P + (int64_t)(c0 + cc + k + b) * a.D, col, a.D, v4));
+                for (; k < nn; ++k) {
+                    const float2 p = load2(a.P + (int64_t)(c0 + cc + k + b) * a.D, col, a.D, v2);
+                    h.x = fmaf(f_s[k], p.x, h.x);
+                    h.y = fmaf(f_s[k], p.y, h.y);
+                }
             }
         }
-        h.x *= inv; h.y *= inv; h.z *= inv; h.w *= inv;
+        h.x *= inv;
+        h.y *= inv;
     }
     if (in) {
         float* out = a.pooled + (int64_t)b * a.D;
-        if (v4) *reinterpret_cast<float4*>(out + col) = h;
+        if (v2) *reinterpret_cast<float2*>(out + col) = h;
         else {
             out[col] = h.x;
             if (col + 1 < a.D) out[col + 1] = h.y;
-            if (col + 2 < a.D) out[col + 2] = h.z;
-            if (col + 3 < a.D) out[col + 3] = h.w;
         }
     }
     if (!a.W) return;
-    // partial logits of these columns, kFinBins bins per pass; warp partials in warp order
-    for (int k0 = 0; k0 < a.K; k0 += kFinBins) {
-        float part[kFinBins];
+    // partial logits of these columns, 32 bins per pass: products, reduce-scatter over the
+    // warp (lane l ends with bin l), warp partials added in warp order
+    for (int k0 = 0; k0 < a.K; k0 += 32) {
+        float part[32];
 #pragma unroll
-        for (int j = 0; j < kFinBins; ++j) {
+        for (int j = 0; j < 32; ++j) {
             if (k0 > 0)
-                wv[j] = k0 + j < a.K && in ? load4(a.W + (int64_t)(k0 + j) * a.D, col, a.D, v4)
-                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+                wv[j] = k0 + j < a.K && in ? load2(a.W + (int64_t)(k0 + j) * a.D, col, a.D, v2)
+                                           : make_float2(0.f, 0.f);
+            part[j] = fmaf(wv[j].x, h.x, wv[j].y * h.y);
         }
-#pragma unroll
-        for (int j = 0; j < kFinBins; ++j) {
-            part[j] = fmaf(wv[j].x, h.x, fmaf(wv[j].y, h.y, fmaf(wv[j].z, h.z, wv[j].w * h.w)));
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) part[j] += __shfl_xor_sync(0xffffffffu, part[j], off);
-        }
-        if (lane == 0)
-#pragma unroll
-            for (int j = 0; j < kFinBins; ++j) red[wid][j] = part[j];
+        red[wid][lane] = warp_reduce_scatter32(part);
         __syncthreads();
-        if (tid < kFinBins && k0 + tid < a.K) {
+        if (tid < 32 && k0 + tid < a.K) {
             float zk = 0.f;
             for (int w = 0; w < nw; ++w) zk += red[w][tid];
             a.zpart[((int64_t)b * a.n_cb + cb) * a.K + k0 + tid] = zk;
@@ -411,15 +418,14 @@ estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int
         }
         ctx->pool_done_cap = B;
     }
-    // workspace: [valid][MZ slots][zpart B x n_cb x K][P slots x D], G + B slots
+    // workspace: [MZ slots][zpart B x n_cb x K][P slots x D], G + B slots
     const int64_t slots = G + B;
-    const size_t off_mz = 256;
+    const size_t off_mz = 0;
     const size_t off_z = align_up(off_mz + sizeof(float2) * (size_t)slots, 256);
     const size_t off_p = align_up(off_z + sizeof(float) * (size_t)B * n_cb * K, 256);
     estp_status s = ws_reserve(ctx, off_p + sizeof(float) * (size_t)slots * (size_t)D);
     if (s != ESTP_OK) return s;
     char* ws = static_cast<char*>(ctx->ws);
-    a.valid = reinterpret_cast<int*>(ws);
     a.MZ = reinterpret_cast<float2*>(ws + off_mz);
     a.P = reinterpret_cast<float*>(ws + off_p);
     dim3 grid((unsigned)G, (unsigned)n_slices);
@@ -428,14 +434,13 @@ estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int
     FinishArgs f{};
     f.P = a.P;
     f.MZ = a.MZ;
-    f.valid = a.valid;
     f.cu = cu;
     f.B = B;
     f.sumT = sumT;
     f.G = a.G;
     f.D = D;
     f.n_cb = n_cb;
-    f.vec4 = D % 4 == 0 && aligned16(pooled) && (!with_head || aligned16(head->W));
+    f.vec2 = D % 2 == 0 && aligned16(pooled) && (!with_head || aligned16(head->W));
     f.pooled = pooled;
     if (with_head) {
         f.done = ctx->pool_done;

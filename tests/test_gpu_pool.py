@@ -113,3 +113,27 @@ def test_head_bins(cuda_lib, K, with_bias):
     P_ref = oracle.pool(hid, H.astype(np.float64), S.astype(np.float64), cu, 0.7, 0.3, 1.0)
     assert_pooled(pooled.cpu().numpy(), P_ref)
     assert_pred(pred.cpu().numpy(), oracle.length_head(P_ref, Wt, b if with_bias else None, c))
+
+
+def test_pool_bad_cu_then_good(cuda_lib):
+    """Bad cu_seqlens (checked on the device): the call records ESTP_ERR_INVALID_ARG and
+    writes nothing else, so the next call on the same context is exact."""
+    cu, hid, H, S, hd = _inputs(synth.BF16, [300, 77, 1500, 9], 3584)
+    Wt, b, c = _head(32, 3584)
+    head = cuda_lib.Head(torch.from_numpy(Wt).cuda(), torch.from_numpy(b).cuda(),
+                         torch.from_numpy(c).cuda())
+    ctx = cuda_lib.Context(0)
+    Hd, Sd = torch.from_numpy(H).cuda(), torch.from_numpy(S).cuda()
+    for bad in ([0, 300, 200, 1877, 1886],    # decreasing
+                [0, 300, 377, 1877, 1885],    # cu[B] != sumT
+                [5, 300, 377, 1877, 1886]):   # cu[0] != 0
+        with pytest.raises(cuda_lib.EstpError) as ei:
+            ctx.pool(hd, Hd, Sd, torch.as_tensor(np.asarray(bad, np.int32), device="cuda"),
+                     0.7, 0.3, 1.0, head=head)
+            ctx.sync_status()
+        assert ei.value.status == cuda_lib.ESTP_ERR_INVALID_ARG
+    pooled, pred = ctx.pool(hd, Hd, Sd, torch.as_tensor(cu, device="cuda"), 0.7, 0.3, 1.0, head=head)
+    ctx.sync_status()
+    P_ref = oracle.pool(hid, H.astype(np.float64), S.astype(np.float64), cu, 0.7, 0.3, 1.0)
+    assert_pooled(pooled.cpu().numpy(), P_ref)
+    assert_pred(pred.cpu().numpy(), oracle.length_head(P_ref, Wt, b, c))
