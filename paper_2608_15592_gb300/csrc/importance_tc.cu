@@ -58,17 +58,16 @@ struct Cfg {
     static constexpr int kAtoms = D / 64;
     static constexpr int kTileBytes = kTile * 128 * kAtoms;  // 128 rows x D bf16
     static constexpr int kStages = D == 64 ? 6 : 2;
-    static constexpr int kKSteps = D / 16;
     // dynamic smem layout (offsets from a 1024-aligned base)
     static constexpr int kFixOff = 0;                               // [2 buffers][A, B]
     static constexpr int kRingOff = 4 * kTileBytes;
     static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][64] f32
     static constexpr int kMergeOff = kNlOff + kEpiWarps * 64 * 4;   // [2][A, B][4][32] float2
     static constexpr int kBarOff = kMergeOff + 2 * 2 * 4 * 32 * 8;
-    // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[kAccBufs], drain,
+    // fix_full/empty[2], ring_full/empty[kStages][kAtoms], acc_full/empty[kAccBufs], drain,
     // sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
     static constexpr int kNumBars =
-        2 + 2 + 2 * kStages + 2 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
+        2 + 2 + 2 * kStages * kAtoms + 2 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
     static constexpr int kLseOff = (kMiscOff + 16 + 4 * kSched + 127) / 128 * 128;  // lse ring
     static constexpr int kSmemBytes = kLseOff + kLseSlots * kLseSlotBytes + 1024;  // + alignment slack
@@ -206,24 +205,43 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
     return t;
 }
 
-// Streamed tile of step s of an item: (head for TMA y, first row).
+// Streamed tiles of an item, step by step: TMA head coordinate y, first row, the query
+// head of the tile and (column sums) its query tile.  Column-sum steps run over the
+// item's query tiles for each selected head of the group in turn; the counters advance
+// without divisions or per-step table lookups.
 template <int MODE>
-__device__ __forceinline__ void step_tile(const TcArgs& a, const TcItem& t, int s, int& y, int& row0,
-                                          int& head, int& qt) {
-    if (MODE == kModeLse) {
-        y = t.h / (a.Hq / a.Hkv);
-        row0 = s * kTile;  // key tile s
-        head = t.h;
-        qt = t.qt0;
-    } else {
-        const int nq = t.qt1 - t.qt0;
-        const int hi = s / nq;
-        qt = t.qt0 + (s - hi * nq);
-        head = a.hs.head_list[a.hs.begin[t.g] + hi];
-        y = head;
-        row0 = qt * kTile;
+struct StepIter {
+    int y, row0, head, qt;
+    int hi;  // column sums: index of the head within the group
+
+    __device__ __forceinline__ StepIter(const TcArgs& a, const TcItem& t) {
+        if (MODE == kModeLse) {
+            head = t.h;
+            y = t.h / (a.Hq / a.Hkv);
+            qt = t.qt0;
+            row0 = 0;  // key tile 0
+        } else {
+            hi = 0;
+            head = a.hs.head_list[a.hs.begin[t.g]];
+            y = head;
+            qt = t.qt0;
+            row0 = qt * kTile;
+        }
     }
-}
+    __device__ __forceinline__ void next(const TcArgs& a, const TcItem& t) {
+        if (MODE == kModeLse) {
+            row0 += kTile;
+        } else if (++qt < t.qt1) {
+            row0 += kTile;
+        } else {
+            qt = t.qt0;
+            row0 = qt * kTile;
+            ++hi;
+            if (hi < a.hs.begin[t.g + 1] - a.hs.begin[t.g]) head = a.hs.head_list[a.hs.begin[t.g] + hi];
+            y = head;
+        }
+    }
+};
 
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -240,9 +258,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::kBarOff);
     uint64_t* fix_full = bars;                    // [2]
     uint64_t* fix_empty = bars + 2;               // [2]
-    uint64_t* ring_full = bars + 4;               // [kStages]
-    uint64_t* ring_empty = bars + 4 + C::kStages; // [kStages]
-    uint64_t* acc_full = bars + 4 + 2 * C::kStages;
+    // ring barriers per (stage, 64-column K atom): the atoms of a stage are refilled as
+    // soon as the MMAs that read them are done
+    uint64_t* ring_full = bars + 4;                             // [kStages][kAtoms]
+    uint64_t* ring_empty = ring_full + C::kStages * C::kAtoms;  // [kStages][kAtoms]
+    uint64_t* acc_full = ring_empty + C::kStages * C::kAtoms;
     uint64_t* acc_empty = acc_full + kAccBufs;
     uint64_t* drain = acc_empty + kAccBufs;
     uint64_t* sched_full = drain + 1;             // [kSched]
@@ -266,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&acc_full[i], 1);
             mbar_init(&acc_empty[i], kEpiWarps);  // one arrival per epilogue warp
         }
-        for (int i = 0; i < C::kStages; ++i) {
+        for (int i = 0; i < C::kStages * C::kAtoms; ++i) {
             mbar_init(&ring_full[i], 1);
             mbar_init(&ring_empty[i], 1);
         }
@@ -345,15 +365,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     &fix_full[fb]);
                 ++n_items;
                 bool ok = true;
-                for (int s = 0; s < t.n_steps; ++s, ++step) {
+                StepIter<MODE> si(a, t);
+                for (int s = 0; s < t.n_steps; ++s, ++step, si.next(a, t)) {
                     const int stage = (int)(step % C::kStages);
                     const uint32_t u = step / C::kStages;
-                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
-                    int y, row0, head, qt;
-                    step_tile<MODE>(a, t, s, y, row0, head, qt);
+                    const int y = si.y, row0 = si.row0, head = si.head;
                     if (MODE == kModeImp) {  // the tile's lse values, from a 16-byte boundary
                         const int ls = (int)(step % kLseSlots);
                         const uint32_t lu = step / kLseSlots;
@@ -366,19 +382,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tma_load_1d(lse_ring + ls * (kLseSlotBytes / 4), &tm_lse, (int)(x & ~int64_t(3)),
                                     &lse_full[ls]);
                     }
-                    mbar_expect_tx(&ring_full[stage], C::kTileBytes);
+                    // ring barriers: one group per K atom (column sums) or one per stage
+                    constexpr int kGroups = MODE == kModeImp ? C::kAtoms : 1;
+                    constexpr int kAtPerGroup = C::kAtoms / kGroups;
 #pragma unroll
-                    for (int at = 0; at < C::kAtoms; ++at)
-                        tma_load_3d(ring + stage * C::kTileBytes + at * kTile * 128, &tm_str, at * 64, y,
-                                    (int)(t.t0 + row0), &ring_full[stage]);
+                    for (int gr = 0; gr < kGroups; ++gr) {
+                        uint64_t* gfull = &ring_full[stage * C::kAtoms + gr];
+                        if (u >= 1 && !wait_bar(&ring_empty[stage * C::kAtoms + gr], (u - 1) & 1, abort_flag,
+                                                a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_expect_tx(gfull, C::kTileBytes / kGroups);
+#pragma unroll
+                        for (int k = 0; k < kAtPerGroup; ++k) {
+                            const int at = gr * kAtPerGroup + k;
+                            tma_load_3d(ring + stage * C::kTileBytes + at * kTile * 128, &tm_str, at * 64, y,
+                                        (int)(t.t0 + row0), gfull);
+                        }
+                    }
+                    if (!ok) break;
                 }
                 if (!ok) break;
                 item = (int)gridDim.x + atomicAdd(&info->next, 1);
             }
             // Every copy this thread issued has landed before the CTA can exit (on the
             // normal path the consumers already waited for all of them).
+            // (a step broken off between atoms left its later atoms unissued; the earlier
+            // ones are waited for with the step's phase)
             for (uint32_t st = 0; st < (uint32_t)C::kStages && st < step; ++st)
-                drain_wait(&ring_full[st], ((step - 1 - st) / C::kStages) & 1, a.status);
+                for (int gr = 0; gr < (MODE == kModeImp ? C::kAtoms : 1); ++gr)
+                    drain_wait(&ring_full[st * C::kAtoms + gr], ((step - 1 - st) / C::kStages) & 1, a.status);
             if (MODE == kModeImp)
                 for (uint32_t ls = 0; ls < (uint32_t)kLseSlots && ls < step; ++ls)
                     drain_wait(&lse_full[ls], ((step - 1 - ls) / kLseSlots) & 1, a.status);
@@ -403,24 +437,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t u = step / C::kStages;
                     const int ab = (int)(step % kAccBufs);
                     const uint32_t ua = step / kAccBufs;
-                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status) ||
-                        (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status))) {
+                    if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
-                    tc_fence_after();
                     const uint32_t str_addr = smem_u32(ring + stage * C::kTileBytes);
+                    // Column sums release each K atom as soon as its MMAs are done; the row
+                    // normaliser, whose single MMA thread is its critical path, keeps one
+                    // barrier per stage.
+                    constexpr int kGroups = MODE == kModeImp ? C::kAtoms : 1;
+                    constexpr int kAtPerGroup = C::kAtoms / kGroups;
 #pragma unroll
-                    for (int kk = 0; kk < C::kKSteps; ++kk) {
-                        const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
-                        const uint64_t sdesc = sw128_desc(str_addr + off);
+                    for (int gr = 0; gr < kGroups; ++gr) {
+                        if (!wait_bar(&ring_full[stage * C::kAtoms + gr], u & 1, abort_flag, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
 #pragma unroll
-                        for (int tau = 0; tau < 2; ++tau)
-                            mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
-                                     sw128_desc(fix_addr + tau * C::kTileBytes + off), sdesc,
-                                     kk > 0 ? 1u : 0u);
+                        for (int k = 0; k < 4 * kAtPerGroup; ++k) {  // the group's K steps of 16
+                            const int kk = gr * 4 * kAtPerGroup + k;
+                            const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
+                            const uint64_t sdesc = sw128_desc(str_addr + off);
+#pragma unroll
+                            for (int tau = 0; tau < 2; ++tau)
+                                mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
+                                         sw128_desc(fix_addr + tau * C::kTileBytes + off), sdesc,
+                                         kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(&ring_empty[stage * C::kAtoms + gr]);
                     }
-                    mma_commit(&ring_empty[stage]);
+                    if (!ok) break;
                     mma_commit(&acc_full[ab]);
                     issued = true;
                 }
@@ -448,9 +495,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const TcItem t = make_item<MODE>(a, item);
             float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
             float m = -1e30f, ssum = 0.f;          // LSE mode
+            StepIter<MODE> si(a, t);
             auto do_step = [&](int s) -> bool {
-                int y, row0, head, qt;
-                step_tile<MODE>(a, t, s, y, row0, head, qt);
+                const int row0 = si.row0, head = si.head, qt = si.qt;
                 if (MODE == kModeImp) {  // -log2e * lse of this warp's 64 query columns
                     const int ls = (int)(step % kLseSlots);
                     if (!warp_wait(&lse_full[ls], (step / kLseSlots) & 1, abort_flag, a.status))
@@ -554,7 +601,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++step;
                 return true;
             };
-            for (int s = 0; s < t.n_steps; ++s)
+            for (int s = 0; s < t.n_steps; ++s, si.next(a, t))
                 if (!(ok = do_step(s))) break;
             if (!ok) break;
             // merge the two column halves of each row (bounded mbarrier hand-off), then write
