@@ -64,10 +64,10 @@ struct Cfg {
     static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][64] f32
     static constexpr int kMergeOff = kNlOff + kEpiWarps * 64 * 4;   // [2][A, B][4][32] float2
     static constexpr int kBarOff = kMergeOff + 2 * 2 * 4 * 32 * 8;
-    // fix_full/empty[2], ring_full/empty[kStages][kAtoms], acc_full/empty[kAccBufs], drain,
-    // sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
+    // fix_full/empty[2], ring_full/empty[kStages][kAtoms], acc_full/empty[A, B][kAccBufs],
+    // drain, sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
     static constexpr int kNumBars =
-        2 + 2 + 2 * kStages * kAtoms + 2 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
+        2 + 2 + 2 * kStages * kAtoms + 4 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
     static constexpr int kLseOff = (kMiscOff + 16 + 4 * kSched + 127) / 128 * 128;  // lse ring
     static constexpr int kSmemBytes = kLseOff + kLseSlots * kLseSlotBytes + 1024;  // + alignment slack
@@ -263,8 +263,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* ring_full = bars + 4;                             // [kStages][kAtoms]
     uint64_t* ring_empty = ring_full + C::kStages * C::kAtoms;  // [kStages][kAtoms]
     uint64_t* acc_full = ring_empty + C::kStages * C::kAtoms;
-    uint64_t* acc_empty = acc_full + kAccBufs;
-    uint64_t* drain = acc_empty + kAccBufs;
+    uint64_t* acc_empty = acc_full + 2 * kAccBufs;   // [A, B][kAccBufs], like acc_full
+    uint64_t* drain = acc_empty + 2 * kAccBufs;
     uint64_t* sched_full = drain + 1;             // [kSched]
     uint64_t* sched_empty = sched_full + kSched;  // [kSched]
     uint64_t* xfull = sched_empty + kSched;       // [2][A, B][4]: half-1 partials ready
@@ -282,9 +282,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&fix_full[i], 1);
             mbar_init(&fix_empty[i], 1);
         }
-        for (int i = 0; i < kAccBufs; ++i) {
+        for (int i = 0; i < 2 * kAccBufs; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], kEpiWarps);  // one arrival per epilogue warp
+            // one arrival per epilogue warp of the tile (column sums) or of both tiles
+            mbar_init(&acc_empty[i], MODE == kModeImp ? kEpiWarps / 2 : kEpiWarps);
         }
         for (int i = 0; i < C::kStages * C::kAtoms; ++i) {
             mbar_init(&ring_full[i], 1);
@@ -437,26 +438,45 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t u = step / C::kStages;
                     const int ab = (int)(step % kAccBufs);
                     const uint32_t ua = step / kAccBufs;
-                    if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
                     const uint32_t str_addr = smem_u32(ring + stage * C::kTileBytes);
-                    // Column sums release each K atom as soon as its MMAs are done; the row
-                    // normaliser, whose single MMA thread is its critical path, keeps one
-                    // barrier per stage.
                     constexpr int kGroups = MODE == kModeImp ? C::kAtoms : 1;
-                    constexpr int kAtPerGroup = C::kAtoms / kGroups;
 #pragma unroll
-                    for (int gr = 0; gr < kGroups; ++gr) {
-                        if (!wait_bar(&ring_full[stage * C::kAtoms + gr], u & 1, abort_flag, a.status)) {
+                    for (int gr = 0; gr < kGroups; ++gr)
+                        if (ok && !wait_bar(&ring_full[stage * C::kAtoms + gr], u & 1, abort_flag, a.status))
+                            ok = false;
+                    if (!ok) break;
+                    if (MODE == kModeImp) {
+                        // tile A's MMAs, then tile B's, each committed on its own accumulator
+                        // barrier: the epilogue of A starts while B's MMAs run, and A's next
+                        // MMAs wait only for A's epilogue
+#pragma unroll
+                        for (int tau = 0; tau < 2; ++tau) {
+                            if (ua >= 1 &&
+                                !wait_bar(&acc_empty[tau * kAccBufs + ab], (ua - 1) & 1, abort_flag, a.status)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+#pragma unroll
+                            for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {  // K steps of 16
+                                const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
+                                mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
+                                         sw128_desc(fix_addr + tau * C::kTileBytes + off),
+                                         sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
+                            }
+                            mma_commit(&acc_full[tau * kAccBufs + ab]);
+                        }
+                        if (!ok) break;
+                    } else {
+                        // the row normaliser's single MMA thread is its critical path: both
+                        // tiles interleaved under one accumulator barrier
+                        if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
 #pragma unroll
-                        for (int k = 0; k < 4 * kAtPerGroup; ++k) {  // the group's K steps of 16
-                            const int kk = gr * 4 * kAtPerGroup + k;
+                        for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {
                             const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
                             const uint64_t sdesc = sw128_desc(str_addr + off);
 #pragma unroll
@@ -465,10 +485,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                          sw128_desc(fix_addr + tau * C::kTileBytes + off), sdesc,
                                          kk > 0 ? 1u : 0u);
                         }
-                        mma_commit(&ring_empty[stage * C::kAtoms + gr]);
+                        mma_commit(&acc_full[ab]);
                     }
-                    if (!ok) break;
-                    mma_commit(&acc_full[ab]);
+#pragma unroll
+                    for (int gr = 0; gr < kGroups; ++gr) mma_commit(&ring_empty[stage * C::kAtoms + gr]);
                     issued = true;
                 }
                 if (!ok) break;
@@ -514,7 +534,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
                 const int ab = (int)(step % kAccBufs);
-                if (!warp_wait(&acc_full[ab], (step / kAccBufs) & 1, abort_flag, a.status))
+                const int abar = (MODE == kModeImp ? tau * kAccBufs : 0) + ab;  // accumulator barrier
+                if (!warp_wait(&acc_full[abar], (step / kAccBufs) & 1, abort_flag, a.status))
                     return false;
                 tc_fence_after();
                 const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) +
@@ -538,7 +559,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (ch == 1) {
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                        if (lane == 0) mbar_arrive(&acc_empty[abar]);
                     }
                     const int cb = col0 + ch * 32;  // tile column of v[0]
                     const float* nc = nl + ch * 32;
