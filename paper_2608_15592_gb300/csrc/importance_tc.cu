@@ -4,16 +4,20 @@
 // and never materialise the attention matrix A (Sec. 3.1).  One persistent CTA per
 // SM works on "pair items": two fixed 128-row tiles (2p and 2p+1) multiplied by the
 // same sequence of streamed 128-row tiles, so that every streamed tile feeds two MMAs.
-// (Tile loads through TMA reach only ~24-34 B/clk per SM; one 128 x 128 x 128 MMA per
-// streamed tile would need ~58.)  The CTA runs a warp-specialised pipeline:
+// The CTA runs a warp-specialised pipeline:
 //   warp 0       TMA producer: the item's two fixed tiles, then a ring of streamed tiles
 //                (128B-swizzled, one 64-column atom per TMA box) and, for column sums,
 //                the lse values of each streamed query tile
-//   warp 1       MMA issuer: D_A = A x S^T and D_B = B x S^T (M = 128 each, N = 128,
-//                fp32 in TMEM), double-buffered: 2 x 2 x 128 = all 512 TMEM columns
+//   warps 1, 18  MMA issuers, one per fixed tile: D_A = A x S^T (warp 1) and
+//                D_B = B x S^T (warp 18), M = 128, N = 128, fp32 in TMEM, each
+//                double-buffered: 2 x 2 x 128 = all 512 TMEM columns
 //   warps 2-17   epilogue: warps 2-9 read D_A, warps 10-17 D_B; warp w reads TMEM lanes
 //                32*(w%4).. (its quarter), and two warps of a quarter split the 128
 //                columns (halves); tcgen05.ld, exp2 and row reductions
+// Two issuers because the tensor core's instruction queue is shallow: a check of an
+// mbarrier costs an issuing thread ~150-180 cycles even when the phase has completed,
+// and with a single issuer the pipe idles through its two waits and commits per step;
+// with one issuer per tile those waits overlap the other tile's MMAs.
 //
 // LSE mode (rows = queries): pair p = query tiles 2p, 2p+1 of one head, streaming the
 //   key tiles 0..2p+1 with a running max (flash-style normaliser); a tile skips the
@@ -40,7 +44,10 @@ constexpr int kPair = 2 * kTile;       // rows of the fixed pair (the plan's til
 constexpr int kQcPair = 2;             // pairs of query tiles per column-sum item
 constexpr int kEpiWarp0 = 2;           // warps 2..17
 constexpr int kEpiWarps = 16;          // 8 per fixed tile
-constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
+// MMA issuers: warp 1 for fixed tile A, warp 18 for tile B, so that one issuer's barrier
+// waits and commits overlap the other's MMAs in the tensor pipe
+constexpr int kMmaWarpB = kEpiWarp0 + kEpiWarps;
+constexpr int kThreads = 32 * (kMmaWarpB + 1);
 constexpr int kAccCols = 128;
 constexpr int kAccBufs = 2;            // accumulator pairs in TMEM (kAccBufs x 2 x 128 columns)
 constexpr int kSched = 4;              // depth of the item-index ring (producer -> consumers)
@@ -64,10 +71,10 @@ struct Cfg {
     static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][64] f32
     static constexpr int kMergeOff = kNlOff + kEpiWarps * 64 * 4;   // [2][A, B][4][32] float2
     static constexpr int kBarOff = kMergeOff + 2 * 2 * 4 * 32 * 8;
-    // fix_full/empty[2], ring_full/empty[kStages][kAtoms], acc_full/empty[A, B][kAccBufs],
-    // drain, sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
+    // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[A, B][kAccBufs],
+    // drain[A, B], sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
     static constexpr int kNumBars =
-        2 + 2 + 2 * kStages * kAtoms + 4 * kAccBufs + 1 + 2 * kSched + 32 + 2 * kLseSlots;
+        2 + 2 + 2 * kStages + 4 * kAccBufs + 2 + 2 * kSched + 32 + 2 * kLseSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
     static constexpr int kLseOff = (kMiscOff + 16 + 4 * kSched + 127) / 128 * 128;  // lse ring
     static constexpr int kSmemBytes = kLseOff + kLseSlots * kLseSlotBytes + 1024;  // + alignment slack
@@ -258,14 +265,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::kBarOff);
     uint64_t* fix_full = bars;                    // [2]
     uint64_t* fix_empty = bars + 2;               // [2]
-    // ring barriers per (stage, 64-column K atom): the atoms of a stage are refilled as
-    // soon as the MMAs that read them are done
-    uint64_t* ring_full = bars + 4;                             // [kStages][kAtoms]
-    uint64_t* ring_empty = ring_full + C::kStages * C::kAtoms;  // [kStages][kAtoms]
-    uint64_t* acc_full = ring_empty + C::kStages * C::kAtoms;
+    uint64_t* ring_full = bars + 4;               // [kStages]
+    uint64_t* ring_empty = ring_full + C::kStages;  // [kStages]
+    uint64_t* acc_full = ring_empty + C::kStages;
     uint64_t* acc_empty = acc_full + 2 * kAccBufs;   // [A, B][kAccBufs], like acc_full
-    uint64_t* drain = acc_empty + 2 * kAccBufs;
-    uint64_t* sched_full = drain + 1;             // [kSched]
+    uint64_t* drain = acc_empty + 2 * kAccBufs;   // [A, B]
+    uint64_t* sched_full = drain + 2;             // [kSched]
     uint64_t* sched_empty = sched_full + kSched;  // [kSched]
     uint64_t* xfull = sched_empty + kSched;       // [2][A, B][4]: half-1 partials ready
     uint64_t* xempty = xfull + 16;                // [2][A, B][4]: half-0 has read them
@@ -280,21 +285,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&fix_full[i], 1);
-            mbar_init(&fix_empty[i], 1);
+            mbar_init(&fix_empty[i], 2);  // both issuers
         }
         for (int i = 0; i < 2 * kAccBufs; ++i) {
             mbar_init(&acc_full[i], 1);
-            // one arrival per epilogue warp of the tile (column sums) or of both tiles
-            mbar_init(&acc_empty[i], MODE == kModeImp ? kEpiWarps / 2 : kEpiWarps);
+            mbar_init(&acc_empty[i], kEpiWarps / 2);  // one arrival per epilogue warp of the tile
         }
-        for (int i = 0; i < C::kStages * C::kAtoms; ++i) {
+        for (int i = 0; i < C::kStages; ++i) {
             mbar_init(&ring_full[i], 1);
-            mbar_init(&ring_empty[i], 1);
+            mbar_init(&ring_empty[i], 2);  // both issuers
         }
-        mbar_init(drain, 1);
+        mbar_init(&drain[0], 1);
+        mbar_init(&drain[1], 1);
         for (int i = 0; i < kSched; ++i) {
             mbar_init(&sched_full[i], 1);
-            mbar_init(&sched_empty[i], 1 + kEpiWarps);  // MMA thread + epilogue warps
+            mbar_init(&sched_empty[i], 2 + kEpiWarps);  // MMA issuers + epilogue warps
         }
         for (int i = 0; i < 16; ++i) {
             mbar_init(&xfull[i], 1);
@@ -383,25 +388,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tma_load_1d(lse_ring + ls * (kLseSlotBytes / 4), &tm_lse, (int)(x & ~int64_t(3)),
                                     &lse_full[ls]);
                     }
-                    // ring barriers: one group per K atom (column sums) or one per stage
-                    constexpr int kGroups = MODE == kModeImp ? C::kAtoms : 1;
-                    constexpr int kAtPerGroup = C::kAtoms / kGroups;
-#pragma unroll
-                    for (int gr = 0; gr < kGroups; ++gr) {
-                        uint64_t* gfull = &ring_full[stage * C::kAtoms + gr];
-                        if (u >= 1 && !wait_bar(&ring_empty[stage * C::kAtoms + gr], (u - 1) & 1, abort_flag,
-                                                a.status)) {
-                            ok = false;
-                            break;
-                        }
-                        mbar_expect_tx(gfull, C::kTileBytes / kGroups);
-#pragma unroll
-                        for (int k = 0; k < kAtPerGroup; ++k) {
-                            const int at = gr * kAtPerGroup + k;
-                            tma_load_3d(ring + stage * C::kTileBytes + at * kTile * 128, &tm_str, at * 64, y,
-                                        (int)(t.t0 + row0), gfull);
-                        }
+                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
                     }
+                    mbar_expect_tx(&ring_full[stage], C::kTileBytes);
+#pragma unroll
+                    for (int at = 0; at < C::kAtoms; ++at)
+                        tma_load_3d(ring + stage * C::kTileBytes + at * kTile * 128, &tm_str, at * 64, y,
+                                    (int)(t.t0 + row0), &ring_full[stage]);
                     if (!ok) break;
                 }
                 if (!ok) break;
@@ -409,19 +404,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // Every copy this thread issued has landed before the CTA can exit (on the
             // normal path the consumers already waited for all of them).
-            // (a step broken off between atoms left its later atoms unissued; the earlier
-            // ones are waited for with the step's phase)
             for (uint32_t st = 0; st < (uint32_t)C::kStages && st < step; ++st)
-                for (int gr = 0; gr < (MODE == kModeImp ? C::kAtoms : 1); ++gr)
-                    drain_wait(&ring_full[st * C::kAtoms + gr], ((step - 1 - st) / C::kStages) & 1, a.status);
+                drain_wait(&ring_full[(step - 1 - st) % C::kStages], ((step - 1 - st) / C::kStages) & 1,
+                           a.status);
             if (MODE == kModeImp)
                 for (uint32_t ls = 0; ls < (uint32_t)kLseSlots && ls < step; ++ls)
                     drain_wait(&lse_full[ls], ((step - 1 - ls) / kLseSlots) & 1, a.status);
             for (int fb = 0; fb < 2 && fb < n_items; ++fb)
                 drain_wait(&fix_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
         }
-    } else if (warp == 1) {
-        // ---------------------------------------------------------- MMA issuer
+    } else if (warp == 1 || warp == kMmaWarpB) {
+        // --------------------------------------------- MMA issuers (tile A, tile B)
+        const int tau = warp == 1 ? 0 : 1;
         if (lane == 0) {
             uint32_t step = 0;
             bool issued = false;
@@ -431,7 +425,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
-                const uint32_t fix_addr = smem_u32(fix + fb * 2 * C::kTileBytes);  // tile A; B follows
+                const uint32_t fix_addr = smem_u32(fix + (fb * 2 + tau) * C::kTileBytes);
                 bool ok = true;
                 for (int s = 0; s < t.n_steps; ++s, ++step) {
                     const int stage = (int)(step % C::kStages);
@@ -439,67 +433,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int ab = (int)(step % kAccBufs);
                     const uint32_t ua = step / kAccBufs;
                     const uint32_t str_addr = smem_u32(ring + stage * C::kTileBytes);
-                    constexpr int kGroups = MODE == kModeImp ? C::kAtoms : 1;
-#pragma unroll
-                    for (int gr = 0; gr < kGroups; ++gr)
-                        if (ok && !wait_bar(&ring_full[stage * C::kAtoms + gr], u & 1, abort_flag, a.status))
-                            ok = false;
-                    if (!ok) break;
-                    if (MODE == kModeImp) {
-                        // tile A's MMAs, then tile B's, each committed on its own accumulator
-                        // barrier: the epilogue of A starts while B's MMAs run, and A's next
-                        // MMAs wait only for A's epilogue
-#pragma unroll
-                        for (int tau = 0; tau < 2; ++tau) {
-                            if (ua >= 1 &&
-                                !wait_bar(&acc_empty[tau * kAccBufs + ab], (ua - 1) & 1, abort_flag, a.status)) {
-                                ok = false;
-                                break;
-                            }
-                            tc_fence_after();
-#pragma unroll
-                            for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {  // K steps of 16
-                                const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
-                                mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
-                                         sw128_desc(fix_addr + tau * C::kTileBytes + off),
-                                         sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
-                            }
-                            mma_commit(&acc_full[tau * kAccBufs + ab]);
-                        }
-                        if (!ok) break;
-                    } else {
-                        // the row normaliser's single MMA thread is its critical path: both
-                        // tiles interleaved under one accumulator barrier
-                        if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-#pragma unroll
-                        for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {
-                            const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
-                            const uint64_t sdesc = sw128_desc(str_addr + off);
-#pragma unroll
-                            for (int tau = 0; tau < 2; ++tau)
-                                mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols),
-                                         sw128_desc(fix_addr + tau * C::kTileBytes + off), sdesc,
-                                         kk > 0 ? 1u : 0u);
-                        }
-                        mma_commit(&acc_full[ab]);
+                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
                     }
-#pragma unroll
-                    for (int gr = 0; gr < kGroups; ++gr) mma_commit(&ring_empty[stage * C::kAtoms + gr]);
+                    if (ua >= 1 && !wait_bar(&acc_empty[tau * kAccBufs + ab], (ua - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
                     issued = true;
+#pragma unroll
+                    for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {  // K steps of 16
+                        const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
+                        mma_bf16(tmem + (uint32_t)((ab * 2 + tau) * kAccCols), sw128_desc(fix_addr + off),
+                                 sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(&acc_full[tau * kAccBufs + ab]);
+                    mma_commit(&ring_empty[stage]);
                 }
                 if (!ok) break;
                 mma_commit(&fix_empty[fb]);
             }
             if (issued) {  // every MMA done before the TMEM is released
-                mma_commit(drain);
-                drain_wait(drain, 0, a.status);
+                mma_commit(&drain[tau]);
+                drain_wait(&drain[tau], 0, a.status);
             }
         }
-    } else {
+    } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
         // ------------------------------------------------------------- epilogue
         const int e = warp - kEpiWarp0;
         const int tau = e >> 3;                    // fixed tile: 0 = A, 1 = B
@@ -534,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
                 const int ab = (int)(step % kAccBufs);
-                const int abar = (MODE == kModeImp ? tau * kAccBufs : 0) + ab;  // accumulator barrier
+                const int abar = tau * kAccBufs + ab;  // accumulator barrier
                 if (!warp_wait(&acc_full[abar], (step / kAccBufs) & 1, abort_flag, a.status))
                     return false;
                 tc_fence_after();
