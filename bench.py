@@ -48,7 +48,9 @@ def _peaks():
 
 # --------------------------------------------------------------------- clocks
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+    """nvidia-smi clocks and throttle reasons, sampled every 50 ms. Each line is stamped
+    with the host time at which it was read, and the summary keeps the lines that fall
+    inside the window set by `window(t0, t1)` (the timed region)."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -56,12 +58,13 @@ class ClockSampler:
 
     def __init__(self, index: int):
         self.index, self.lines, self.proc = index, [], None
+        self.t0, self.t1 = None, None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -71,7 +74,10 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
+
+    def window(self, t0: float, t1: float):
+        self.t0, self.t1 = t0, t1
 
     def __exit__(self, *exc):
         if self.proc:
@@ -85,7 +91,11 @@ class ClockSampler:
     def summary(self):
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        lines = self.lines
+        if self.t0 is not None:
+            # a line is read up to one sampling interval after the sample was taken
+            lines = [x for x in lines if self.t0 <= x[0] <= self.t1 + 0.05]
+        for _, ln in lines:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 9:
                 continue
@@ -254,11 +264,14 @@ def run_ours(args, rank, world, local_rank):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local_rank) as clk:
+        time.sleep(0.3)  # nvidia-smi is sampling before the timed region starts
+        t_host0 = time.time()
         start.record()
         for k in range(K):
             st.run(ev_steps[k])
         end.record()
         torch.cuda.synchronize()
+        clk.window(t_host0, time.time())
     if world > 1:
         torch.distributed.barrier()
     st.ctx.sync_status()
