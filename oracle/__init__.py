@@ -9,7 +9,7 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   attn_lse        the row normaliser of the causal softmax A (Sec. 3.1)
   attn_colsum     sum_i A_ij of Eq. 2-0 for one layer, summed over query heads
   attn_colsum_rows  the same from the rows i >= row_from only (exact for late keys)
-  importance      Eq. 2-0: S_j = C_j / (N * layers * heads)
+  importance      Eq. 2-0: S_j = C_j / (N * layers * heads); divisor variants of its 1/N
   pool            Eqs. 2-2, 2-3, 2-4
   length_head     Eq. 3-2 with a linear projection
 
@@ -55,6 +55,7 @@ class _Lib:
             "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
             "oracle_attn_colsum_rows": [P, P, I, I, I, I, D, P, I, P, I, I, I64, P, I],
             "oracle_importance": [P, P, I, I, I, P],
+            "oracle_importance_div": [P, P, I, I, I, I, I, P],
             "oracle_pool": [P, I, I64, I64, P, P, P, I, D, D, D, P, P],
             "oracle_length_head": [P, I, I64, P, P, P, I, P, P],
         }
@@ -192,12 +193,22 @@ def attn_colsum_rows(Q, K, cu_seqlens, scale, row_from: int, heads=None, exclude
     return out
 
 
-def importance(C, cu_seqlens, n_layers: int, n_heads: int) -> np.ndarray:
-    """Eq. 2-0 scaling of accumulated column sums."""
+DIVISORS = {"length": 0, "causal": 1, "none": 2}
+
+
+def importance(C, cu_seqlens, n_layers: int, n_heads: int, divisor: str = "length",
+               exclude_self: bool = False) -> np.ndarray:
+    """Eq. 2-0 scaling of accumulated column sums. divisor: "length" (the paper's N),
+    "causal" (the queries whose terms enter C_j) or "none" (mean column sum)."""
     C, cu = np.ascontiguousarray(C, dtype=np.float64), _cu(cu_seqlens)
     out = np.zeros_like(C)
-    _check(_load().oracle_importance(_ptr(C), _ptr(cu), len(cu) - 1, n_layers, n_heads,
-                                     _ptr(out)), "importance")
+    if divisor == "length":
+        _check(_load().oracle_importance(_ptr(C), _ptr(cu), len(cu) - 1, n_layers, n_heads,
+                                         _ptr(out)), "importance")
+    else:
+        _check(_load().oracle_importance_div(_ptr(C), _ptr(cu), len(cu) - 1, n_layers, n_heads,
+                                             DIVISORS[divisor], int(bool(exclude_self)),
+                                             _ptr(out)), "importance")
     return out
 
 

@@ -257,11 +257,26 @@ int oracle_attn_colsum(const void* Q, const void* K, int dtype, int Hq, int Hkv,
 
 int oracle_importance(const double* C, const int32_t* cu_seqlens, int B, int n_layers,
                       int n_heads, double* S_out) {
+    return oracle_importance_div(C, cu_seqlens, B, n_layers, n_heads, ORACLE_DIV_LENGTH, 0, S_out);
+}
+
+/* Eq. 2-0 with the divisor of the column sum chosen: the prompt length N (the paper),
+ * the number of queries whose terms enter C_j (rows i >= j, or i > j without the
+ * diagonal; S_j = 0 when there are none), or 1. */
+int oracle_importance_div(const double* C, const int32_t* cu_seqlens, int B, int n_layers,
+                          int n_heads, int divisor, int exclude_self, double* S_out) {
     if (!valid_cu(cu_seqlens, B) || n_layers <= 0 || n_heads <= 0) return -1;
+    if (divisor != ORACLE_DIV_LENGTH && divisor != ORACLE_DIV_CAUSAL && divisor != ORACLE_DIV_NONE)
+        return -1;
     for (int b = 0; b < B; ++b) {
         int64_t t0 = cu_seqlens[b], N = (int64_t)cu_seqlens[b + 1] - cu_seqlens[b];
-        for (int64_t j = 0; j < N; ++j)
-            S_out[t0 + j] = C[t0 + j] / ((double)N * (double)n_layers * (double)n_heads);
+        for (int64_t j = 0; j < N; ++j) {
+            double n;
+            if (divisor == ORACLE_DIV_LENGTH) n = (double)N;
+            else if (divisor == ORACLE_DIV_CAUSAL) n = (double)(N - j - (exclude_self ? 1 : 0));
+            else n = 1.0;
+            S_out[t0 + j] = n > 0.0 ? C[t0 + j] / (n * (double)n_layers * (double)n_heads) : 0.0;
+        }
     }
     return 0;
 }

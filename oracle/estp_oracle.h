@@ -13,6 +13,7 @@
  *   oracle_attn_lse            log-normaliser of the softmax rows of A (Sec. 3.1)
  *   oracle_attn_colsum         the column sums of A inside Eq. 2-0 (Sec. 3.1)
  *   oracle_importance          Eq. 2-0 (the 1/N scaling and the head/layer mean)
+ *   oracle_importance_div      Eq. 2-0 with the causal-count or no divisor (variants)
  *   oracle_pool                Eqs. 2-2, 2-3, 2-4 (Sec. 3.2)
  *   oracle_length_head         Eq. 3-2 (Sec. 3.3), linear projection + softmax
  *
@@ -71,6 +72,15 @@ int oracle_attn_colsum_rows(const void* Q, const void* K, int dtype, int Hq, int
  * N_b is the length of the prompt that holds token j.  S_out: [sumT]. */
 int oracle_importance(const double* C, const int32_t* cu_seqlens, int B, int n_layers,
                       int n_heads, double* S_out);
+
+/* Variants of Eq. 2-0's divisor (not printed in the paper):
+ *   ORACLE_DIV_LENGTH  N_b (= oracle_importance)
+ *   ORACLE_DIV_CAUSAL  the causal count n_j = N_b - j (N_b - j - 1 with exclude_self):
+ *                      the queries whose terms enter C_j; S_j = 0 where n_j = 0
+ *   ORACLE_DIV_NONE    1: S_j = C_j / (n_layers * n_heads), the mean column sum */
+enum { ORACLE_DIV_LENGTH = 0, ORACLE_DIV_CAUSAL = 1, ORACLE_DIV_NONE = 2 };
+int oracle_importance_div(const double* C, const int32_t* cu_seqlens, int B, int n_layers,
+                          int n_heads, int divisor, int exclude_self, double* S_out);
 
 /* Eqs. 2-2..2-4 per prompt b:  T_i = lambda1*S_i + lambda2*H_i,
  * e_i = exp(T_i/alpha) / sum_j exp(T_j/alpha) over the prompt's tokens,

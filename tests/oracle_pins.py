@@ -182,6 +182,51 @@ def pin_importance_uniform_harmonic():
             _close(S[cu[b]:cu[b + 1]], ref, rtol=1e-12, what="harmonic")
 
 
+def pin_importance_divisors_uniform():
+    """The divisor variants of Eq. 2-0 under uniform causal rows (Q = 0), A_ij = 1/(i+1):
+    C_j = H_N - H_j (H_N - H_{j+1} without the diagonal).  Causal count: n_j = N - j
+    (N - j - 1 without the diagonal, S = 0 where it is 0); none: S_j = C_j."""
+    rng = _rng(15)
+    cu = np.asarray([0, 1, 9, 200], dtype=np.int32)
+    Q, K = _qk(rng, cu, 2, 1, 16)
+    for excl in (False, True):
+        C = oracle.attn_colsum(np.zeros_like(Q), K, cu, 0.25, exclude_self=excl)
+        Sc = oracle.importance(C, cu, n_layers=1, n_heads=2, divisor="causal", exclude_self=excl)
+        Sn = oracle.importance(C, cu, n_layers=1, n_heads=2, divisor="none", exclude_self=excl)
+        for b in range(len(cu) - 1):
+            N = int(cu[b + 1] - cu[b])
+            Hn = np.concatenate([[0.0], np.cumsum(1.0 / np.arange(1, N + 1))])
+            j = np.arange(N)
+            col = Hn[N] - Hn[j + (1 if excl else 0)]
+            cnt = N - j - (1 if excl else 0)
+            ref_c = np.where(cnt > 0, col / np.maximum(cnt, 1), 0.0)
+            _close(Sc[cu[b]:cu[b + 1]], ref_c, rtol=1e-12, what=f"causal excl={excl}")
+            _close(Sn[cu[b]:cu[b + 1]], col, rtol=1e-12, what=f"none excl={excl}")
+
+
+def pin_importance_divisor_invariants():
+    """Random inputs: with the diagonal, every softmax row sums to 1, so the "none"
+    variant sums to N_b per prompt; the causal variant of the last token is its own
+    diagonal weight A_{N-1,N-1} averaged over heads, 1 / sum_j exp(s_{N-1,j} - s_{N-1,N-1})
+    from a direct softmax of that row."""
+    rng = _rng(16)
+    cu = np.asarray([0, 5, 64, 130], dtype=np.int32)
+    Hq, Hkv, d, sc = 4, 2, 16, 0.3
+    Q, K = _qk(rng, cu, Hq, Hkv, d)
+    C = oracle.attn_colsum(Q, K, cu, sc)
+    Sn = oracle.importance(C, cu, n_layers=1, n_heads=Hq, divisor="none")
+    Sc = oracle.importance(C, cu, n_layers=1, n_heads=Hq, divisor="causal")
+    q64, k64 = Q.astype(np.float64), K.astype(np.float64)
+    for b in range(len(cu) - 1):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        _close(np.sum(Sn[t0:t1]), float(t1 - t0), rtol=1e-12, what="none sums to N")
+        diag = 0.0
+        for h in range(Hq):
+            s = sc * (k64[t0:t1, h // (Hq // Hkv)] @ q64[t1 - 1, h])
+            diag += 1.0 / np.sum(np.exp(s - s[-1]))
+        _close(Sc[t1 - 1], diag / Hq, rtol=1e-12, what="causal last token")
+
+
 def pin_importance_gqa_and_scale():
     """GQA: query head h reads KV head h // rep -- equal to the MHA case with K heads
     repeated; the softmax scale multiplies the scores (doubling Q == doubling scale)."""

@@ -26,9 +26,14 @@ MUTANTS = [
     ("lse sign", "m + log(Z);", "m - log(Z);"),
     ("rows_from off by one", "for (int64_t i = c->row_from; i < T; ++i) {",
      "for (int64_t i = c->row_from + 1; i < T; ++i) {"),
-    ("causal count divisor", "((double)N * (double)n_layers",
-     "((double)(N - j) * (double)n_layers"),
-    ("head mean dropped", "(double)n_layers * (double)n_heads)", "(double)n_layers)"),
+    ("causal count divisor", "if (divisor == ORACLE_DIV_LENGTH) n = (double)N;",
+     "if (divisor == ORACLE_DIV_LENGTH) n = (double)(N - j);"),
+    ("head mean dropped", "(n * (double)n_layers * (double)n_heads)", "(n * (double)n_layers)"),
+    ("causal count keeps the diagonal", "(double)(N - j - (exclude_self ? 1 : 0))",
+     "(double)(N - j)"),
+    ("causal count off by one", "(double)(N - j - (exclude_self ? 1 : 0))",
+     "(double)(N - j + 1 - (exclude_self ? 1 : 0))"),
+    ("no-divisor variant divides by N", "else n = 1.0;", "else n = (double)N;"),
     ("temperature ignored", "w[i] = T / alpha;", "w[i] = T;"),
     ("lambdas swapped", "lambda1 * S[t0 + i] + lambda2 * H[t0 + i]",
      "lambda1 * H[t0 + i] + lambda2 * S[t0 + i]"),
