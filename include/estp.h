@@ -134,9 +134,22 @@ estp_status estp_attn_lse(estp_ctx* ctx, const void* Q, const void* K, estp_dtyp
  *   lse   : fp32 [Hq, sumT] from estp_attn_lse / the prefill, or NULL to have
  *           the library compute it (into the workspace) first.
  *   heads : HOST int32 [n_heads] query-head indices in [0, Hq), or NULL = all Hq.
- *   flags : 0, or ESTP_IMP_EXCLUDE_SELF to drop the diagonal term A_jj from C_j
- *           (the softmax rows keep it). */
+ *   flags : OR of
+ *     ESTP_IMP_EXCLUDE_SELF  drop the diagonal term A_jj from C_j (the softmax rows keep
+ *                            it); Sec. 3.1 speaks of attention from all *other* tokens.
+ *     ESTP_IMP_DIV_CAUSAL    finalize divides C_j by the causal count n_j (the queries
+ *                            whose terms enter C_j: N_b - j, or N_b - j - 1 with
+ *                            ESTP_IMP_EXCLUDE_SELF; S_j = 0 where n_j = 0) instead of N_b.
+ *     ESTP_IMP_DIV_NONE      finalize divides by nothing but the layer/head count: the
+ *                            mean column sum, N_b times the S_j of Eq. 2-0.
+ *           The two divisor flags are variants of Eq. 2-0's 1/N, not printed in the
+ *           paper; at most one may be set.  They take effect in
+ *           estp_attn_importance_finalize and are fixed by the call that opens the
+ *           accumulation (accumulate = 0): later calls of it must pass the same divisor
+ *           flags, and with ESTP_IMP_DIV_CAUSAL the same ESTP_IMP_EXCLUDE_SELF. */
 #define ESTP_IMP_EXCLUDE_SELF 1u
+#define ESTP_IMP_DIV_CAUSAL 2u
+#define ESTP_IMP_DIV_NONE 4u
 estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
                                  estp_dtype dtype, const float* lse, int32_t Hq, int32_t Hkv,
                                  int32_t head_dim, float softmax_scale, const int32_t* heads,
@@ -146,8 +159,10 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
 
 /* Ends an accumulation: importance_out[j] = C_j / (N_b * n_layers * n_heads), N_b
  * the length of the prompt holding token j (Eq. 2-0's 1/N, then the mean over the
- * selected layers and heads).  n_layers = number of estp_attn_importance calls the
- * caller means to average over (normally the calls since accumulate = 0).
+ * selected layers and heads); N_b is replaced by the causal count n_j, or by 1, when
+ * the accumulation was opened with ESTP_IMP_DIV_CAUSAL or ESTP_IMP_DIV_NONE.
+ * n_layers = number of estp_attn_importance calls the caller means to average over
+ * (normally the calls since accumulate = 0).
  *   importance_out : fp32 [sumT]. */
 estp_status estp_attn_importance_finalize(estp_ctx* ctx, int32_t n_layers,
                                           float* importance_out, estp_stream_t stream);

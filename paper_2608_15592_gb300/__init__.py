@@ -28,6 +28,9 @@ ESTP_OK, ESTP_ERR_INVALID_ARG, ESTP_ERR_UNSUPPORTED = 0, 1, 2
 ESTP_ERR_CUDA, ESTP_ERR_TIMEOUT, ESTP_ERR_WORKSPACE = 3, 4, 5
 ESTP_F32, ESTP_BF16 = 0, 1
 ESTP_IMP_EXCLUDE_SELF = 1
+ESTP_IMP_DIV_CAUSAL = 2
+ESTP_IMP_DIV_NONE = 4
+_DIVISOR_FLAGS = {"length": 0, "causal": ESTP_IMP_DIV_CAUSAL, "none": ESTP_IMP_DIV_NONE}
 
 # every entry point declared in include/estp.h
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
@@ -170,8 +173,10 @@ class Context:
 
     def attn_importance(self, Q, K, cu_seqlens, max_seqlen: int, lse=None,
                         scale: float | None = None, heads=None, accumulate: bool = False,
-                        exclude_self: bool = False, stream=None):
-        """estp_attn_importance for one layer (column sums into the context)."""
+                        exclude_self: bool = False, divisor: str = "length", stream=None):
+        """estp_attn_importance for one layer (column sums into the context).
+        divisor: "length" (Eq. 2-0's 1/N), "causal" or "none" (ESTP_IMP_DIV_*), applied
+        by attn_importance_finalize and fixed by the call that opens the accumulation."""
         sumT, Hq, d = Q.shape
         Hkv = K.shape[1]
         scale = 1.0 / math.sqrt(d) if scale is None else scale
@@ -184,7 +189,8 @@ class Context:
                                         Hkv, d, scale, hp, nh, _ptr(cu_seqlens),
                                         cu_seqlens.numel() - 1, sumT, max_seqlen,
                                         1 if accumulate else 0,
-                                        ESTP_IMP_EXCLUDE_SELF if exclude_self else 0,
+                                        (ESTP_IMP_EXCLUDE_SELF if exclude_self else 0)
+                                        | _DIVISOR_FLAGS[divisor],
                                         _stream(stream)))
 
     def attn_importance_finalize(self, n_layers: int, sumT: int, device=None, out=None,

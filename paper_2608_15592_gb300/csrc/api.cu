@@ -205,7 +205,10 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
     estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
                                 B, sumT, max_seqlen);
     if (st != ESTP_OK) return st;
-    if (flags & ~ESTP_IMP_EXCLUDE_SELF) return fail(ESTP_ERR_INVALID_ARG, "unknown flags");
+    constexpr uint32_t kDiv = ESTP_IMP_DIV_CAUSAL | ESTP_IMP_DIV_NONE;
+    if (flags & ~(ESTP_IMP_EXCLUDE_SELF | kDiv)) return fail(ESTP_ERR_INVALID_ARG, "unknown flags");
+    if ((flags & kDiv) == kDiv)
+        return fail(ESTP_ERR_INVALID_ARG, "ESTP_IMP_DIV_CAUSAL and ESTP_IMP_DIV_NONE together");
     ImpHeads hs;
     st = build_heads(heads, n_heads, Hq, Hkv, &hs);
     if (st != ESTP_OK) return st;
@@ -216,6 +219,12 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
             ctx->imp_n_heads != hs.n_heads)
             return fail(ESTP_ERR_INVALID_ARG,
                         "accumulate=1 with different cu_seqlens/B/sumT/head count");
+        // the finalize divisor is fixed when the accumulation opens; the causal count
+        // also depends on whether the self term is summed
+        const uint32_t fixed = (ctx->imp_flags & ESTP_IMP_DIV_CAUSAL) ? (kDiv | ESTP_IMP_EXCLUDE_SELF) : kDiv;
+        if ((flags & fixed) != (ctx->imp_flags & fixed))
+            return fail(ESTP_ERR_INVALID_ARG,
+                        "accumulate=1 with divisor flags that differ from the opening call");
     }
     if (lse && !aligned16(lse)) return fail(ESTP_ERR_INVALID_ARG, "lse must be 16-byte aligned");
     st = set_device(ctx);
@@ -238,6 +247,7 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
     ctx->imp_B = B;
     ctx->imp_cu = cu_seqlens;
     ctx->imp_n_heads = hs.n_heads;
+    if (!accumulate) ctx->imp_flags = flags;
     if (sumT == 0 || B == 0) return ESTP_OK;
     return launch_importance(ctx, Q, K, dtype, lse, Hq, Hkv, head_dim, softmax_scale, hs,
                              cu_seqlens, B, sumT, max_seqlen, accumulate != 0, flags,
@@ -254,7 +264,7 @@ estp_status estp_attn_importance_finalize(estp_ctx* ctx, int32_t n_layers,
     estp_status st = set_device(ctx);
     if (st != ESTP_OK) return st;
     return launch_importance_finalize(ctx, ctx->imp_acc, ctx->imp_cu, ctx->imp_B, ctx->imp_sumT,
-                                      n_layers, ctx->imp_n_heads, importance_out,
+                                      n_layers, ctx->imp_n_heads, ctx->imp_flags, importance_out,
                                       reinterpret_cast<cudaStream_t>(stream));
 }
 

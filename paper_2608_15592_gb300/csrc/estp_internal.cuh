@@ -21,6 +21,7 @@ struct estp_ctx {
     int32_t imp_B = 0;
     const int32_t* imp_cu = nullptr;
     int32_t imp_n_heads = 0;
+    uint32_t imp_flags = 0;     // flags of the opening call (divisor variant, self term)
     uint32_t* pool_done = nullptr;      // per-prompt arrival counters of the pooling kernel
     int32_t pool_done_cap = 0;
 };
@@ -101,8 +102,8 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
                               cudaStream_t st);
 
 estp_status launch_importance_finalize(estp_ctx* ctx, const float* acc, const int32_t* cu, int B,
-                                       int64_t sumT, int n_layers, int n_heads, float* out,
-                                       cudaStream_t st);
+                                       int64_t sumT, int n_layers, int n_heads, uint32_t flags,
+                                       float* out, cudaStream_t st);
 
 estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int64_t D,
                         int64_t ldh, const float* H, const float* S, const int32_t* cu, int B,

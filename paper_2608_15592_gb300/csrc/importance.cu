@@ -290,15 +290,20 @@ __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const
     acc[j] = accumulate ? acc[j] + v : v;
 }
 
+// S_j = C_j / (n_j * layers * heads): n_j = N_b (Eq. 2-0), the causal count of the
+// queries whose terms enter C_j (div 1: N_b - j, one fewer without the diagonal;
+// S_j = 0 where it is 0), or 1 (div 2).
 __global__ void imp_finalize_kernel(const float* acc, const int32_t* cu, int B, int64_t sumT,
-                                    float inv_lh, float* out) {
+                                    float inv_lh, int div, int exclude_self, float* out) {
     __shared__ int32_t cu_s[kCuStage];
     const int32_t* cuv = stage_cu(cu, B, cu_s);
     const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= sumT) return;
     const int b = upper_slot(cuv, B, j);
-    const float N = (float)(cuv[b + 1] - cuv[b]);
-    out[j] = acc[j] * inv_lh / N;
+    int64_t n = cuv[b + 1] - cuv[b];
+    if (div == 1) n = (int64_t)cuv[b + 1] - j - (exclude_self ? 1 : 0);
+    else if (div == 2) n = 1;
+    out[j] = n > 0 ? acc[j] * inv_lh / (float)n : 0.f;
 }
 
 size_t simt_smem(int d, bool with_lse) {
@@ -419,11 +424,13 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
 }
 
 estp_status launch_importance_finalize(estp_ctx* ctx, const float* acc, const int32_t* cu, int B,
-                                       int64_t sumT, int n_layers, int n_heads, float* out,
-                                       cudaStream_t st) {
+                                       int64_t sumT, int n_layers, int n_heads, uint32_t flags,
+                                       float* out, cudaStream_t st) {
     (void)ctx;
     const float inv_lh = 1.f / ((float)n_layers * (float)n_heads);
-    imp_finalize_kernel<<<(unsigned)((sumT + 255) / 256), 256, 0, st>>>(acc, cu, B, sumT, inv_lh, out);
+    const int div = (flags & ESTP_IMP_DIV_CAUSAL) ? 1 : (flags & ESTP_IMP_DIV_NONE) ? 2 : 0;
+    imp_finalize_kernel<<<(unsigned)((sumT + 255) / 256), 256, 0, st>>>(
+        acc, cu, B, sumT, inv_lh, div, (flags & ESTP_IMP_EXCLUDE_SELF) ? 1 : 0, out);
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "finalize launch");
 }

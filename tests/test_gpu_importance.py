@@ -42,7 +42,8 @@ def _qk(w, cu, layer):
     return Qh, Kh, Qd, Kd
 
 
-def _run(cuda_lib, w, cu, layers, heads=None, exclude_self=False, supply_lse=False):
+def _run(cuda_lib, w, cu, layers, heads=None, exclude_self=False, supply_lse=False,
+         divisor="length"):
     ctx = cuda_lib.Context(0)
     cu_d = torch.as_tensor(cu, device="cuda")
     maxT = int(np.diff(cu).max())
@@ -55,13 +56,13 @@ def _run(cuda_lib, w, cu, layers, heads=None, exclude_self=False, supply_lse=Fal
             lse = torch.as_tensor(oracle.attn_lse(Qh, Kh, cu, 1 / math.sqrt(w.d)),
                                   dtype=torch.float32, device="cuda").contiguous()
         ctx.attn_importance(Qd, Kd, cu_d, maxT, lse=lse, heads=heads, accumulate=n > 0,
-                            exclude_self=exclude_self)
+                            exclude_self=exclude_self, divisor=divisor)
         oracle.attn_colsum(Qh, Kh, cu, 1 / math.sqrt(w.d), heads=heads,
                            exclude_self=exclude_self, out=C)
     S = ctx.attn_importance_finalize(len(layers), sumT)
     ctx.sync_status()
     nh = w.Hq if heads is None else len(heads)
-    ref = oracle.importance(C, cu, len(layers), nh)
+    ref = oracle.importance(C, cu, len(layers), nh, divisor=divisor, exclude_self=exclude_self)
     return S.cpu().numpy(), ref
 
 
@@ -142,6 +143,48 @@ def test_importance_device_checks(cuda_lib):
     fresh.attn_importance(Qd, Kd, cu_d, 100)
     with pytest.raises(cuda_lib.EstpError):  # a different prompt set cannot join it
         fresh.attn_importance(Qd[:100], Kd[:100], cu_d[:2], 100, accumulate=True)
+
+
+@pytest.mark.parametrize("divisor", ["causal", "none"])
+@pytest.mark.parametrize("exclude_self", [False, True])
+@pytest.mark.parametrize("dtype", [synth.BF16, synth.F32])
+def test_importance_divisor_variants(cuda_lib, dtype, divisor, exclude_self):
+    """The divisor variants of Eq. 2-0 (ESTP_IMP_DIV_CAUSAL / _NONE) against the oracle:
+    1-token and empty prompts (a zero causal count without the diagonal), several tiles,
+    a head subset and two layers."""
+    w, cu = _wl(dtype, [1, 0, 257, 40, 130], 8, 2, 128 if dtype == synth.BF16 else 64, layers=3)
+    S, ref = _run(cuda_lib, w, cu, [0, 2], heads=[1, 2, 5, 7], exclude_self=exclude_self,
+                  divisor=divisor)
+    assert_importance(S, ref)
+    if exclude_self and divisor == "causal":  # the last token of every prompt has n_j = 0
+        for b in range(len(cu) - 1):
+            if cu[b + 1] > cu[b]:
+                assert S[cu[b + 1] - 1] == 0.0
+
+
+def test_importance_divisor_flags_checked(cuda_lib):
+    """Both divisor flags at once, and a later call whose divisor (or, under the causal
+    divisor, self-term) flags differ from the opening call's, are refused on the host."""
+    w, cu = _wl(synth.BF16, [70, 30], 4, 2, 64)
+    _, _, Qd, Kd = _qk(w, cu, 0)
+    cu_d = torch.as_tensor(cu, device="cuda")
+    ctx = cuda_lib.Context(0)
+    lib = cuda_lib.lib
+    rc = lib.estp_attn_importance(ctx._h, Qd.data_ptr(), Kd.data_ptr(), 1, None, 4, 2, 64, 0.125,
+                                  None, 4, cu_d.data_ptr(), 2, 100, 70, 0,
+                                  cuda_lib.ESTP_IMP_DIV_CAUSAL | cuda_lib.ESTP_IMP_DIV_NONE, None)
+    assert rc == cuda_lib.ESTP_ERR_INVALID_ARG
+    ctx.attn_importance(Qd, Kd, cu_d, 70, divisor="causal")
+    with pytest.raises(cuda_lib.EstpError):
+        ctx.attn_importance(Qd, Kd, cu_d, 70, accumulate=True)  # length divisor now
+    with pytest.raises(cuda_lib.EstpError):
+        ctx.attn_importance(Qd, Kd, cu_d, 70, accumulate=True, divisor="causal", exclude_self=True)
+    ctx.attn_importance(Qd, Kd, cu_d, 70, accumulate=True, divisor="causal")
+    plain = cuda_lib.Context(0)  # the length divisor lets the self term vary per layer
+    plain.attn_importance(Qd, Kd, cu_d, 70)
+    plain.attn_importance(Qd, Kd, cu_d, 70, accumulate=True, exclude_self=True)
+    ctx.sync_status()
+    plain.sync_status()
 
 
 @pytest.mark.parametrize("w", [W.C1, W.C2], ids=lambda w: w.name)
