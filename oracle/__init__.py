@@ -12,6 +12,7 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   importance      Eq. 2-0: S_j = C_j / (N * layers * heads); divisor variants of its 1/N
   pool            Eqs. 2-2, 2-3, 2-4
   length_head     Eq. 3-2 with a linear projection
+  head_loss       Eqs. 3-1, 3-3 (soft-label CE + MSE) and their gradients
 
 bf16 arrays are passed as numpy uint16 holding the raw bfloat16 bits.
 """
@@ -58,6 +59,7 @@ class _Lib:
             "oracle_importance_div": [P, P, I, I, I, I, I, P],
             "oracle_pool": [P, I, I64, I64, P, P, P, I, D, D, D, P, P],
             "oracle_length_head": [P, I, I64, P, P, P, I, P, P],
+            "oracle_head_loss": [P, I, I64, P, P, P, I, P, D, P, P, P, P],
         }
         for name, args in sig.items():
             fn = getattr(lib, name)
@@ -243,3 +245,23 @@ def length_head(pooled, W, bias, centers, return_probs: bool = False):
     _check(_load().oracle_length_head(_ptr(pooled), B, D, _ptr(W), _ptr(bias), _ptr(centers),
                                       K, _ptr(p), _ptr(y)), "length_head")
     return (y, p) if return_probs else y
+
+
+def head_loss(pooled, W, bias, centers, y, lambda3: float, grads: bool = True):
+    """Eqs. 3-1 and 3-3 through the linear head of Eq. 3-2, batch mean; returns the loss
+    and, if asked, (grad_W [K, D], grad_bias [K], grad_pooled [B, D])."""
+    pooled = np.ascontiguousarray(pooled, dtype=np.float64)
+    B, D = pooled.shape
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    K = W.shape[0]
+    bias = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    centers = np.ascontiguousarray(centers, dtype=np.float32)
+    y = np.ascontiguousarray(y, dtype=np.float32)
+    loss = np.zeros(1, dtype=np.float64)
+    gW = np.zeros((K, D)) if grads else None
+    gb = np.zeros(K) if grads else None
+    gp = np.zeros((B, D)) if grads else None
+    _check(_load().oracle_head_loss(_ptr(pooled), B, D, _ptr(W), _ptr(bias), _ptr(centers), K,
+                                    _ptr(y), float(lambda3), _ptr(loss), _ptr(gW), _ptr(gb),
+                                    _ptr(gp)), "head_loss")
+    return (float(loss[0]), gW, gb, gp) if grads else float(loss[0])

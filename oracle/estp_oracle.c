@@ -344,3 +344,68 @@ int oracle_length_head(const double* pooled, int B, int64_t D, const float* W,
     free(z);
     return 0;
 }
+
+/* -------------------------------------------------------- Eqs. 3-1, 3-3 */
+
+/* Soft label of Eq. 3-1: p_j = exp(-|j - i|) / sum_k exp(-|k - i|), i the bin whose
+ * centre is nearest to y (the lower index on a tie). */
+static int nearest_bin(const float* centers, int K, double y) {
+    int best = 0;
+    double d = fabs(y - (double)centers[0]);
+    for (int k = 1; k < K; ++k) {
+        double e = fabs(y - (double)centers[k]);
+        if (e < d) { d = e; best = k; }
+    }
+    return best;
+}
+
+int oracle_head_loss(const double* pooled, int B, int64_t D, const float* W, const float* bias,
+                     const float* centers, int K, const float* y, double lambda3,
+                     double* loss_out, double* grad_W, double* grad_bias, double* grad_pooled) {
+    if (B <= 0 || D <= 0 || K <= 0 || !pooled || !W || !centers || !y || !loss_out) return -1;
+    double* ph = (double*)malloc(sizeof(double) * (size_t)B * K);
+    double* yh = (double*)malloc(sizeof(double) * (size_t)B);
+    double* dz = (double*)malloc(sizeof(double) * (size_t)K);
+    if (oracle_length_head(pooled, B, D, W, bias, centers, K, ph, yh) != 0) {
+        free(ph); free(yh); free(dz);
+        return -1;
+    }
+    if (grad_W) for (int64_t q = 0; q < (int64_t)K * D; ++q) grad_W[q] = 0.0;
+    if (grad_bias) for (int k = 0; k < K; ++k) grad_bias[k] = 0.0;
+    double ce = 0.0, mse = 0.0;
+    for (int b = 0; b < B; ++b) {
+        const double* p_hat = ph + (int64_t)b * K;
+        const int i = nearest_bin(centers, K, (double)y[b]);
+        double norm = 0.0;
+        for (int k = 0; k < K; ++k) norm += exp(-fabs((double)(k - i)));
+        const double err = yh[b] - (double)y[b];
+        for (int k = 0; k < K; ++k) {
+            const double p = exp(-fabs((double)(k - i))) / norm;
+            ce -= p * log(p_hat[k]);
+            /* d/dz_k of the batch mean: CE term p_hat_k - p_k (sum_k p_k = 1); MSE term
+             * 2 (y_hat - y) dy_hat/dz_k with dy_hat/dz_k = p_hat_k (c_k - y_hat) */
+            dz[k] = (lambda3 * (p_hat[k] - p) +
+                     (1.0 - lambda3) * 2.0 * err * p_hat[k] * ((double)centers[k] - yh[b])) / (double)B;
+        }
+        mse += err * err;
+        const double* h = pooled + (int64_t)b * D;
+        for (int k = 0; k < K; ++k) {
+            double* gw = grad_W ? grad_W + (int64_t)k * D : NULL;  /* row k of dL/dW */
+            if (grad_bias) grad_bias[k] += dz[k];
+            if (gw)
+                for (int64_t x = 0; x < D; ++x) gw[x] += dz[k] * h[x];
+        }
+        if (grad_pooled)
+            for (int64_t x = 0; x < D; ++x) {
+                double g = 0.0;
+                for (int k = 0; k < K; ++k) {
+                    const float* wk = W + (int64_t)k * D;  /* row k of the head */
+                    g += (double)wk[x] * dz[k];
+                }
+                grad_pooled[(int64_t)b * D + x] = g;
+            }
+    }
+    *loss_out = lambda3 * ce / (double)B + (1.0 - lambda3) * mse / (double)B;
+    free(ph); free(yh); free(dz);
+    return 0;
+}

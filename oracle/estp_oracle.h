@@ -16,6 +16,7 @@
  *   oracle_importance_div      Eq. 2-0 with the causal-count or no divisor (variants)
  *   oracle_pool                Eqs. 2-2, 2-3, 2-4 (Sec. 3.2)
  *   oracle_length_head         Eq. 3-2 (Sec. 3.3), linear projection + softmax
+ *   oracle_head_loss           Eqs. 3-1 and 3-3 (Sec. 3.3) and their gradients
  *
  * Parity status: every function is pinned by the CPU tests (closed forms,
  * invariants, brute force against independent library routines); none is
@@ -97,6 +98,15 @@ int oracle_pool(const void* hidden, int dtype, int64_t D, int64_t ldh, const dou
 int oracle_length_head(const double* pooled, int B, int64_t D, const float* W,
                        const float* bias, const float* centers, int K, double* probs_out,
                        double* yhat_out);
+
+/* Eqs. 3-1 and 3-3 through the linear head of Eq. 3-2, averaged over the B prompts:
+ *   L = lambda3 * mean_b CE(p_b, p_hat_b) + (1 - lambda3) * mean_b (y_b - y_hat_b)^2,
+ * p_b the soft label of Eq. 3-1 around the bin whose centre is nearest to y_b (lower
+ * index on a tie).  loss_out: [1]; the gradients of L (each may be NULL):
+ * grad_W [K, D], grad_bias [K], grad_pooled [B, D]. */
+int oracle_head_loss(const double* pooled, int B, int64_t D, const float* W, const float* bias,
+                     const float* centers, int K, const float* y, double lambda3,
+                     double* loss_out, double* grad_W, double* grad_bias, double* grad_pooled);
 
 #ifdef __cplusplus
 }

@@ -382,4 +382,99 @@ def pin_head():
     _close(y, ref_p @ c.astype(np.float64), rtol=1e-11, what="expectation")
 
 
+def _soft_label(K, i):
+    """Eq. 3-1 written out: exp(-|j - i|) normalised over the K bins."""
+    e = np.exp(-np.abs(np.arange(K) - i).astype(np.float64))
+    return e / e.sum()
+
+
+def pin_head_loss_closed_forms():
+    """W = 0, bias = 0: p_hat is uniform (1/K) and y_hat the mean centre, so
+    CE = ln K for every target and MSE = (mean c - y)^2; with lambda3 = 1 the loss is
+    ln K exactly and dL/db_k = (1/K - p_k) averaged over the batch."""
+    K, D = 8, 6
+    c = ((np.arange(K) + 0.5) * 100).astype(np.float32)
+    h = _rng(17).standard_normal((3, D))
+    y = np.asarray([40.0, 420.0, 799.0], np.float32)   # bins 0, 4, 7 (nearest centres)
+    Wz, bz = np.zeros((K, D), np.float32), np.zeros(K, np.float32)
+    L1, gW, gb, gp = oracle.head_loss(h, Wz, bz, c, y, 1.0)
+    _close(L1, math.log(K), rtol=1e-13, what="CE of a uniform prediction")
+    ref_gb = np.mean([1.0 / K - _soft_label(K, i) for i in (0, 4, 7)], axis=0)
+    _close(gb, ref_gb, rtol=1e-12, atol=1e-15, what="CE bias gradient")
+    _close(gp, np.zeros_like(gp), what="W = 0: no gradient to the features")
+    L0 = oracle.head_loss(h, Wz, bz, c, y, 0.0, grads=False)
+    mc = float(np.mean(c.astype(np.float64)))
+    _close(L0, float(np.mean((mc - y.astype(np.float64)) ** 2)), rtol=1e-13, what="MSE")
+
+
+def pin_head_loss_soft_label():
+    """A head whose softmax equals the soft label of the target's bin: the CE term is
+    the label's own entropy -sum p ln p (minimum of CE over p_hat), and the label is
+    symmetric, sums to 1 and falls by exactly e per bin away from i."""
+    K, D = 9, 4
+    c = np.arange(K, dtype=np.float32) * 10.0
+    for i in (0, 3, 8):
+        p = _soft_label(K, i)
+        _close(p.sum(), 1.0, rtol=1e-15, what="sums to 1")
+        _close(p[i + 1:] * math.e, p[i:-1], rtol=1e-13, atol=0, what="geometric decay")
+        bias = np.log(p).astype(np.float32)        # softmax(bias) == p up to fp32 rounding
+        h = np.zeros((1, D))
+        y = np.asarray([c[i] + 1.0], np.float32)   # nearest centre: bin i
+        L = oracle.head_loss(h, np.zeros((K, D), np.float32), bias, c, y, 1.0, grads=False)
+        q = special.softmax(bias.astype(np.float64))
+        _close(L, float(-(p * np.log(q)).sum()), rtol=1e-12, what="CE with p_hat = softmax(bias)")
+        _close(L, float(-(p * np.log(p)).sum()), rtol=1e-6, what="CE close to the label entropy")
+
+
+def pin_head_loss_gradients():
+    """The analytic gradients against central finite differences of the oracle's own
+    loss, for W, the bias and the pooled features, at several lambda3."""
+    rng = _rng(18)
+    B, D, K = 3, 5, 6
+    c = ((np.arange(K) + 0.5) * 3).astype(np.float32)
+    h = rng.standard_normal((B, D))
+    W = (0.5 * rng.standard_normal((K, D))).astype(np.float32)
+    b = rng.standard_normal(K).astype(np.float32)
+    y = np.asarray([1.0, 7.9, 16.0], np.float32)
+    for lam in (0.0, 0.3, 1.0):
+        _, gW, gb, gp = oracle.head_loss(h, W, b, c, y, lam)
+        eps = 1e-5
+        num_p = np.zeros_like(h)
+        for idx in np.ndindex(h.shape):
+            hp, hm = h.copy(), h.copy()
+            hp[idx] += eps
+            hm[idx] -= eps
+            num_p[idx] = (oracle.head_loss(hp, W, b, c, y, lam, grads=False) -
+                          oracle.head_loss(hm, W, b, c, y, lam, grads=False)) / (2 * eps)
+        _close(gp, num_p, rtol=1e-6, atol=1e-8, what=f"d/dpooled lam={lam}")
+        # W and b are fp32 parameters: difference them in float64 through an exact
+        # reparametrisation (a feature of value 1 carries the bias, h scaled by W)
+        num_b = np.zeros(K)
+        for k in range(K):
+            bp, bm = b.astype(np.float64).copy(), b.astype(np.float64).copy()
+            bp[k] += 1e-3
+            bm[k] -= 1e-3
+            hx = np.concatenate([h, np.ones((B, 1))], axis=1)
+            Wp = np.concatenate([W, bp[:, None].astype(np.float32)], axis=1)
+            Wm = np.concatenate([W, bm[:, None].astype(np.float32)], axis=1)
+            num_b[k] = (oracle.head_loss(hx, Wp, None, c, y, lam, grads=False) -
+                        oracle.head_loss(hx, Wm, None, c, y, lam, grads=False)) / (
+                            float(np.float32(bp[k])) - float(np.float32(bm[k])))
+        _close(gb, num_b, rtol=2e-3, atol=1e-6, what=f"d/dbias lam={lam}")
+        # W is an fp32 parameter: central differences with the exact fp32 step
+        for k, x in ((0, 0), (2, 3), (5, 4)):
+            Wp, Wm = W.copy(), W.copy()
+            Wp[k, x] = np.float32(W[k, x] + np.float32(1e-3))
+            Wm[k, x] = np.float32(W[k, x] - np.float32(1e-3))
+            num = (oracle.head_loss(h, Wp, b, c, y, lam, grads=False) -
+                   oracle.head_loss(h, Wm, b, c, y, lam, grads=False)) / (float(Wp[k, x]) - float(Wm[k, x]))
+            _close(gW[k, x], num, rtol=2e-3, atol=1e-6, what=f"d/dW[{k},{x}] lam={lam}")
+        # the batch loss is the mean of the per-prompt losses: dW = mean_b dz_b h_b^T
+        ref_gW = np.zeros((K, D))
+        for bb in range(B):
+            _, _, gb1, _ = oracle.head_loss(h[bb:bb + 1], W, b, c, y[bb:bb + 1], lam)
+            ref_gW += np.outer(gb1, h[bb]) / B
+        _close(gW, ref_gW, rtol=1e-12, atol=1e-14, what=f"dW = sum_b dz_b h_b^T lam={lam}")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

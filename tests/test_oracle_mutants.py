@@ -42,6 +42,17 @@ MUTANTS = [
     ("head bias dropped", "double acc = bias ? (double)bias[k] : 0.0;", "double acc = 0.0;"),
     ("head W transposed", "W[(int64_t)k * D + x]", "W[(int64_t)x * K + k]"),
     ("expectation over bin index", "y += p * (double)centers[k];", "y += p * (double)k;"),
+    ("MSE gradient without its factor 2", "(1.0 - lambda3) * 2.0 * err", "(1.0 - lambda3) * err"),
+    ("CE gradient sign", "(lambda3 * (p_hat[k] - p) +", "(lambda3 * (p - p_hat[k]) +"),
+    ("MSE not averaged over the batch", "(1.0 - lambda3) * mse / (double)B;",
+     "(1.0 - lambda3) * mse;"),
+    ("soft label decays with the squared distance",
+     "const double p = exp(-fabs((double)(k - i))) / norm;",
+     "const double p = exp(-(double)((k - i) * (k - i))) / norm;"),
+    ("gradient not divided by the batch size", "((double)centers[k] - yh[b])) / (double)B;",
+     "((double)centers[k] - yh[b]));"),
+    ("feature gradient through W transposed", "g += (double)wk[x] * dz[k];",
+     "g += (double)W[x * K + k] * dz[k];"),
 ]
 
 
