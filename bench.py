@@ -309,6 +309,7 @@ def run_ours(args, rank, world, local_rank):
                 "peak_source": f"{peak_src} ({'hbm_gbs' if dk['bound'] == 'hbm' else 'bf16_tflops_sustained'})"}
 
     e2e = run_e2e(args, st, estp, dev, world)
+    head_loss = time_head_loss(st, dev)
     clocks = clk.summary()
     del st
     if rank != 0:
@@ -326,7 +327,35 @@ def run_ours(args, rank, world, local_rank):
                    "l2": "inputs larger than L2 (~6.4 GB per step), no flush"},
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": st_launches(w) * K, "clocks": clocks,
+        "head_loss": head_loss,
     }
+
+
+def time_head_loss(st, dev, iters: int = 50):
+    """The training loss of the length head (Eqs. 3-1 to 3-3, estp_head_loss) on the
+    step's pooled features with synthetic targets: not part of the step, timed on its
+    own with CUDA events. Its algorithmic bytes (W and the pooled features read by the
+    forward and the gradient kernels, the three gradients written) are a few MB, so it
+    is bound by launch latency, not by HBM."""
+    import torch
+    B, D = st.pooled.shape
+    K = st.head.W.shape[0]
+    g = torch.Generator(device=dev).manual_seed(7)
+    targets = torch.rand(B, generator=g, device=dev) * float(st.head.centers[-1] + st.head.centers[0])
+    for _ in range(3):
+        st.ctx.head_loss(st.pooled, st.head, targets, 0.5)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        st.ctx.head_loss(st.pooled, st.head, targets, 0.5)
+    b.record()
+    torch.cuda.synchronize()
+    st.ctx.sync_status()
+    ms = a.elapsed_time(b) / iters
+    nbytes = 4 * (2 * K * D + 2 * B * D + K * D + K + B * D + B * K)
+    return {"ms": ms, "B": B, "D": D, "K": K, "launches": 2, "bytes": nbytes,
+            "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "launch"}
 
 
 def resident_bytes(w):

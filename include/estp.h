@@ -200,6 +200,30 @@ estp_status estp_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int64
                       estp_mix_params mix, const estp_head* head, float* pooled_out,
                       float* pred_len_out, estp_stream_t stream);
 
+/* ------------------------------------------------------------------ (d)
+ * Training loss of the length head (Sec. 3.3), for fitting W and bias on pooled
+ * features: the soft label of Eq. 3-1,
+ *   p_bj = exp(-|j - i_b|) / sum_k exp(-|k - i_b|),
+ * i_b the bin whose centre is nearest to the target y_b (the lower index on a tie),
+ * the prediction of Eq. 3-2 through the linear head, and the loss of Eq. 3-3 averaged
+ * over the B prompts:
+ *   L = lambda3 * mean_b CE(p_b, p_hat_b) + (1 - lambda3) * mean_b (y_b - y_hat_b)^2,
+ * with CE(p, q) = -sum_k p_k ln q_k, and the gradients of L.
+ *   pooled      : fp32 [B, D] (estp_pool's pooled_out)
+ *   head        : HOST pointer to the head description (W [K, D], bias or NULL, centers)
+ *   targets     : fp32 [B] target lengths y_b
+ *   lambda3     : weight of the cross-entropy term, finite
+ *   loss_out    : fp32 [1]
+ *   grad_W      : fp32 [K, D] dL/dW, or NULL
+ *   grad_bias   : fp32 [K] dL/dbias, or NULL
+ *   grad_pooled : fp32 [B, D] dL/dpooled, or NULL
+ * B >= 1, D >= 1, 1 <= K <= 1024.  Every sum runs in a fixed order (no atomics), so
+ * repeated calls give identical bits.  All arrays are caller-owned device memory. */
+estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                           const estp_head* head, const float* targets, float lambda3,
+                           float* loss_out, float* grad_W, float* grad_bias,
+                           float* grad_pooled, estp_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

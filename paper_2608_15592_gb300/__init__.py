@@ -35,7 +35,8 @@ _DIVISOR_FLAGS = {"length": 0, "causal": ESTP_IMP_DIV_CAUSAL, "none": ESTP_IMP_D
 # every entry point declared in include/estp.h
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
-           "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc")
+           "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
+           "estp_head_loss")
 
 
 class EstpError(RuntimeError):
@@ -76,6 +77,8 @@ def _load():
         "estp_token_entropy_noalloc": ([P, ctypes.c_int, I64, I64, I64, P, P], ctypes.c_int),
         "estp_pool": ([P, P, ctypes.c_int, I64, I64, P, P, P, I32, I64, MixParams,
                        ctypes.POINTER(_Head), P, P, P], ctypes.c_int),
+        "estp_head_loss": ([P, P, I32, I64, ctypes.POINTER(_Head), P, F, P, P, P, P, P],
+                           ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -204,6 +207,23 @@ class Context:
         return out
 
     # ------------------------------------------------------------------ (c)
+    def head_loss(self, pooled, head: Head, targets, lambda3: float, grads: bool = True,
+                  stream=None):
+        """estp_head_loss (Eqs. 3-1 to 3-3): returns (loss [1], and if grads:
+        dL/dW [K, D], dL/dbias [K], dL/dpooled [B, D]), fp32 CUDA tensors."""
+        import torch
+        B, D = pooled.shape
+        K = head.W.shape[0]
+        dev = pooled.device
+        loss = torch.empty(1, dtype=torch.float32, device=dev)
+        gW = torch.empty(K, D, dtype=torch.float32, device=dev) if grads else None
+        gb = torch.empty(K, dtype=torch.float32, device=dev) if grads else None
+        gp = torch.empty(B, D, dtype=torch.float32, device=dev) if grads else None
+        hp = ctypes.pointer(_Head(_ptr(head.W), _ptr(head.bias), _ptr(head.centers), K))
+        _check(lib.estp_head_loss(self._h, _ptr(pooled), B, D, hp, _ptr(targets), lambda3,
+                                  _ptr(loss), _ptr(gW), _ptr(gb), _ptr(gp), _stream(stream)))
+        return (loss, gW, gb, gp) if grads else loss
+
     def pool(self, hidden, entropy, importance, cu_seqlens, lambda1: float, lambda2: float,
              alpha: float, head: Head | None = None, D: int | None = None, pooled=None,
              pred=None, stream=None):

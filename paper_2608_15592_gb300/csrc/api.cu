@@ -295,4 +295,20 @@ estp_status estp_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int64
                        head, pooled_out, pred_len_out, reinterpret_cast<cudaStream_t>(stream));
 }
 
+estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                           const estp_head* head, const float* targets, float lambda3,
+                           float* loss_out, float* grad_W, float* grad_bias,
+                           float* grad_pooled, estp_stream_t stream) {
+    if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
+    if (B < 1 || D < 1) return fail(ESTP_ERR_INVALID_ARG, "need B >= 1 and D >= 1");
+    if (!head || !head->W || !head->centers || head->K < 1 || head->K > 1024)
+        return fail(ESTP_ERR_INVALID_ARG, "head needs W, centers and 1 <= K <= 1024");
+    if (!std::isfinite(lambda3)) return fail(ESTP_ERR_INVALID_ARG, "lambda3 must be finite");
+    if (!pooled || !targets || !loss_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    estp_status st = set_device(ctx);
+    if (st != ESTP_OK) return st;
+    return launch_head_loss(ctx, pooled, B, D, *head, targets, lambda3, loss_out, grad_W,
+                            grad_bias, grad_pooled, reinterpret_cast<cudaStream_t>(stream));
+}
+
 }  // extern "C"

@@ -101,6 +101,10 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
                               int max_seqlen, bool accumulate, uint32_t flags, float* acc,
                               cudaStream_t st);
 
+estp_status launch_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                             const estp_head& head, const float* targets, float lambda3,
+                             float* loss, float* grad_W, float* grad_bias, float* grad_pooled,
+                             cudaStream_t st);
 estp_status launch_importance_finalize(estp_ctx* ctx, const float* acc, const int32_t* cu, int B,
                                        int64_t sumT, int n_layers, int n_heads, uint32_t flags,
                                        float* out, cudaStream_t st);
