@@ -13,6 +13,7 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   pool            Eqs. 2-2, 2-3, 2-4
   length_head     Eq. 3-2 with a linear projection
   head_loss       Eqs. 3-1, 3-3 (soft-label CE + MSE) and their gradients
+  misalignment    the entropy/importance misalignment counts of Sec. 1 (Fig. 1b), numpy
 
 bf16 arrays are passed as numpy uint16 holding the raw bfloat16 bits.
 """
@@ -265,3 +266,32 @@ def head_loss(pooled, W, bias, centers, y, lambda3: float, grads: bool = True):
                                     _ptr(y), float(lambda3), _ptr(loss), _ptr(gW), _ptr(gb),
                                     _ptr(gp)), "head_loss")
     return (float(loss[0]), gW, gb, gp) if grads else float(loss[0])
+
+
+def misalignment(H, S, cu_seqlens, pct: int = 40) -> np.ndarray:
+    """Per prompt b: k = floor(pct * T_b / 100); TopX / BotX the k tokens with the largest /
+    smallest X (ties: the lower token index first), X in {H, S}. Returns int64 [B, 3]:
+    (k, |TopH & BotS|, |BotH & TopS|) -- high-entropy tokens of low importance and
+    low-entropy tokens of high importance (the paper splits at the 60th percentile:
+    pct = 40)."""
+    H = np.asarray(H, dtype=np.float64)
+    S = np.asarray(S, dtype=np.float64)
+    cu = _cu(cu_seqlens)
+    if not 1 <= pct <= 50:
+        raise ValueError("pct must be in 1..50")
+    out = np.zeros((len(cu) - 1, 3), dtype=np.int64)
+    for b in range(len(cu) - 1):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        T = t1 - t0
+        k = pct * T // 100
+        out[b, 0] = k
+        if k == 0:
+            continue
+        idx = np.arange(T)
+        # sort by value, the lower index first among equal values (lexsort: last key primary)
+        top = lambda x: set(np.lexsort((idx, -x))[:k].tolist())
+        bot = lambda x: set(np.lexsort((idx, x))[:k].tolist())
+        h, s = H[t0:t1], S[t0:t1]
+        out[b, 1] = len(top(h) & bot(s))
+        out[b, 2] = len(bot(h) & top(s))
+    return out

@@ -477,4 +477,43 @@ def pin_head_loss_gradients():
         _close(gW, ref_gW, rtol=1e-12, atol=1e-14, what=f"dW = sum_b dz_b h_b^T lam={lam}")
 
 
+def pin_misalignment():
+    """The misalignment counts against sets built from scipy's ordinal ranks (ties by
+    order of appearance, i.e. the lower index first), and the limits: S = H gives 0 and
+    0, S = -H gives k and k, all-tied values pick the k lowest indices for both
+    directions; for independent measures about pct % of TopH lands in BotS."""
+    rng = _rng(19)
+    cu = np.asarray([0, 0, 1, 2, 3, 10, 137, 1137], dtype=np.int32)
+    H = rng.standard_normal(int(cu[-1]))
+    S = rng.standard_normal(int(cu[-1]))
+    H[200:260] = 0.5   # ties inside a prompt
+    S[230:300] = -1.0
+    for pct in (40, 25, 50):
+        got = oracle.misalignment(H, S, cu, pct)
+        for b in range(len(cu) - 1):
+            t0, t1 = int(cu[b]), int(cu[b + 1])
+            k = pct * (t1 - t0) // 100
+            assert got[b, 0] == k
+            if k == 0:
+                assert got[b, 1] == got[b, 2] == 0
+                continue
+            rh_d = stats.rankdata(-H[t0:t1], method="ordinal")   # 1 = largest
+            rh_a = stats.rankdata(H[t0:t1], method="ordinal")    # 1 = smallest
+            rs_d = stats.rankdata(-S[t0:t1], method="ordinal")
+            rs_a = stats.rankdata(S[t0:t1], method="ordinal")
+            assert got[b, 1] == int(np.sum((rh_d <= k) & (rs_a <= k))), (pct, b)
+            assert got[b, 2] == int(np.sum((rh_a <= k) & (rs_d <= k))), (pct, b)
+    same = oracle.misalignment(H, H, cu)
+    assert np.all(same[:, 1] == 0) and np.all(same[:, 2] == 0)
+    anti = oracle.misalignment(H, -H, cu)
+    # S = -H: TopH = BotS exactly when no two H values of a prompt tie
+    distinct = [b for b in range(len(cu) - 1) if len(np.unique(H[cu[b]:cu[b + 1]])) == cu[b + 1] - cu[b]]
+    assert all(anti[b, 1] == anti[b, 0] and anti[b, 2] == anti[b, 0] for b in distinct)
+    flat = oracle.misalignment(np.zeros(20), np.zeros(20), np.asarray([0, 20], np.int32))
+    assert flat.tolist() == [[8, 8, 8]]   # both directions pick tokens 0..7
+    big = oracle.misalignment(rng.standard_normal(50000), rng.standard_normal(50000),
+                              np.asarray([0, 50000], np.int32))
+    assert abs(big[0, 1] / big[0, 0] - 0.4) < 0.02 and abs(big[0, 2] / big[0, 0] - 0.4) < 0.02
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
