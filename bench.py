@@ -310,6 +310,7 @@ def run_ours(args, rank, world, local_rank):
 
     e2e = run_e2e(args, st, estp, dev, world)
     head_loss = time_head_loss(st, dev)
+    misalign = time_misalignment(st)
     clocks = clk.summary()
     del st
     if rank != 0:
@@ -327,7 +328,7 @@ def run_ours(args, rank, world, local_rank):
                    "l2": "inputs larger than L2 (~6.4 GB per step), no flush"},
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": st_launches(w) * K, "clocks": clocks,
-        "head_loss": head_loss,
+        "head_loss": head_loss, "misalignment": misalign,
     }
 
 
@@ -356,6 +357,28 @@ def time_head_loss(st, dev, iters: int = 50):
     nbytes = 4 * (2 * K * D + 2 * B * D + K * D + K + B * D + B * K)
     return {"ms": ms, "B": B, "D": D, "K": K, "launches": 2, "bytes": nbytes,
             "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "launch"}
+
+
+def time_misalignment(st, iters: int = 50):
+    """The entropy/importance misalignment counts (estp_misalignment, pct = 40) on the
+    step's H and S: a diagnostic, timed on its own. One CTA per prompt runs four radix
+    selections (8 passes each over the prompt's values, from L2) and a counting pass;
+    its algorithmic bytes are the 8 bytes per token of H and S."""
+    import torch
+    for _ in range(3):
+        st.ctx.misalignment(st.H, st.S, st.cu)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        st.ctx.misalignment(st.H, st.S, st.cu)
+    b.record()
+    torch.cuda.synchronize()
+    st.ctx.sync_status()
+    ms = a.elapsed_time(b) / iters
+    nbytes = 8 * st.sumT + 12 * st.w.B
+    return {"ms": ms, "B": st.w.B, "tokens": st.sumT, "pct": 40, "launches": 1, "bytes": nbytes,
+            "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "latency (selection passes)"}
 
 
 def resident_bytes(w):

@@ -224,6 +224,22 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
                            float* loss_out, float* grad_W, float* grad_bias,
                            float* grad_pooled, estp_stream_t stream);
 
+/* Entropy/importance misalignment, the diagnostic behind Fig. 1b and Sec. 3.1's
+ * motivation (not part of the predictor).  Per prompt b, with k = floor(pct*T_b/100),
+ * TopX and BotX are the k tokens with the largest and with the smallest X (ties: the
+ * lower token index first) for X = entropy H and importance S:
+ *   counts_out[b] = { k, |TopH ∩ BotS|, |BotH ∩ TopS| }
+ * i.e. high-entropy tokens of low importance and low-entropy tokens of high importance.
+ * The paper splits at the 60th percentile: pct = 40.
+ *   entropy, importance : fp32 [sumT], finite
+ *   pct                 : 1..50
+ *   counts_out          : int32 [B, 3]
+ * Bad cu_seqlens (not non-decreasing from 0 to sumT) record ESTP_ERR_INVALID_ARG in the
+ * status word and write nothing. */
+estp_status estp_misalignment(estp_ctx* ctx, const float* entropy, const float* importance,
+                              const int32_t* cu_seqlens, int32_t B, int64_t sumT, int32_t pct,
+                              int32_t* counts_out, estp_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

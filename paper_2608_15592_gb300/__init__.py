@@ -36,7 +36,7 @@ _DIVISOR_FLAGS = {"length": 0, "causal": ESTP_IMP_DIV_CAUSAL, "none": ESTP_IMP_D
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
            "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
-           "estp_head_loss")
+           "estp_head_loss", "estp_misalignment")
 
 
 class EstpError(RuntimeError):
@@ -79,6 +79,7 @@ def _load():
                        ctypes.POINTER(_Head), P, P, P], ctypes.c_int),
         "estp_head_loss": ([P, P, I32, I64, ctypes.POINTER(_Head), P, F, P, P, P, P, P],
                            ctypes.c_int),
+        "estp_misalignment": ([P, P, P, P, I32, I64, I32, P, P], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -207,6 +208,16 @@ class Context:
         return out
 
     # ------------------------------------------------------------------ (c)
+    def misalignment(self, entropy, importance, cu_seqlens, pct: int = 40, out=None,
+                     stream=None):
+        """estp_misalignment: int32 [B, 3] = (k, |TopH & BotS|, |BotH & TopS|) per prompt."""
+        import torch
+        B = cu_seqlens.numel() - 1
+        out = torch.empty(B, 3, dtype=torch.int32, device=entropy.device) if out is None else out
+        _check(lib.estp_misalignment(self._h, _ptr(entropy), _ptr(importance), _ptr(cu_seqlens),
+                                     B, entropy.numel(), pct, _ptr(out), _stream(stream)))
+        return out
+
     def head_loss(self, pooled, head: Head, targets, lambda3: float, grads: bool = True,
                   stream=None):
         """estp_head_loss (Eqs. 3-1 to 3-3): returns (loss [1], and if grads:

@@ -311,4 +311,20 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
                             grad_bias, grad_pooled, reinterpret_cast<cudaStream_t>(stream));
 }
 
+estp_status estp_misalignment(estp_ctx* ctx, const float* entropy, const float* importance,
+                              const int32_t* cu_seqlens, int32_t B, int64_t sumT, int32_t pct,
+                              int32_t* counts_out, estp_stream_t stream) {
+    if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
+    if (B < 0 || sumT < 0 || sumT > INT32_MAX)
+        return fail(ESTP_ERR_INVALID_ARG, "need B >= 0 and 0 <= sumT < 2^31");
+    if (pct < 1 || pct > 50) return fail(ESTP_ERR_INVALID_ARG, "pct must be in 1..50");
+    if (B == 0) return ESTP_OK;
+    if (!cu_seqlens || !counts_out || (sumT > 0 && (!entropy || !importance)))
+        return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    estp_status st = set_device(ctx);
+    if (st != ESTP_OK) return st;
+    return launch_misalignment(ctx, entropy, importance, cu_seqlens, B, sumT, pct, counts_out,
+                               reinterpret_cast<cudaStream_t>(stream));
+}
+
 }  // extern "C"
