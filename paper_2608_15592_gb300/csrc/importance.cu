@@ -18,6 +18,9 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
                                                          int max_seqlen, int tile, int qc,
                                                          int mult, int kind, int32_t* base,
                                                          PlanInfo* info, int* status) {
+    // the tensor-core kernel that consumes the plan may launch now and run its prologue;
+    // it waits for this grid before its first read of the plan
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     // thread t owns prompts [t*per, (t+1)*per); one read of cu, warp-shuffle scans
     __shared__ int64_t warp_sum[32];
     __shared__ int bad;
@@ -275,6 +278,9 @@ __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const
                                   int accumulate, float* acc) {
     __shared__ int32_t cu_s[kCuStage];
     const int32_t* cuv = stage_cu(cu, B, cu_s);
+    // the partials are complete past this point (launched as a programmatic dependent
+    // of the column-sum kernel; a no-op after an ordinary launch)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= sumT) return;
     float v = 0.f;
@@ -417,8 +423,21 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
         if (dtype == ESTP_BF16) imp_simt_kernel<true><<<grid, kSThreads, smem, st>>>(a);
         else imp_simt_kernel<false><<<grid, kSThreads, smem, st>>>(a);
     }
-    imp_reduce_kernel<<<(unsigned)((sumT + 255) / 256), 256, 0, st>>>(
-        part, info, cu, B, sumT, hs.n_groups, tile, qc, accumulate ? 1 : 0, acc);
+    {  // a programmatic dependent of the column-sum kernel: it waits on it on the device
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)((sumT + 255) / 256));
+        cfg.blockDim = dim3(256);
+        cfg.stream = st;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cudaError_t e = cudaLaunchKernelEx(&cfg, imp_reduce_kernel, (const float*)part,
+                                           (const PlanInfo*)info, cu, B, sumT, hs.n_groups, tile,
+                                           qc, accumulate ? 1 : 0, acc);
+        if (e != cudaSuccess) return cuda_fail(e, "importance reduce launch");
+    }
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "importance launch");
 }

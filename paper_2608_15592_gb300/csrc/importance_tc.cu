@@ -318,10 +318,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                      "r"(kAccBufs * 2 * kAccCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
+    // the column-sum reduce (a programmatic dependent) may launch now; it waits for
+    // this grid before reading the partials
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // the plan (and, in column-sum mode, the lse values) are complete past this point
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     PlanInfo* info = const_cast<PlanInfo*>(a.info);
     const int total = info->total;
 
@@ -680,7 +685,20 @@ estp_status launch_tc(estp_ctx* ctx, const CUtensorMap& fixm, const CUtensorMap&
     const int smem = Cfg<D>::kSmemBytes;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "tc kernel smem attribute");
-    kern<<<ctx->num_sms, kThreads, smem, st>>>(fixm, strm, lsem, a);
+    // a programmatic dependent of the plan kernel: the launch and the prologue (barriers,
+    // TMEM, tensor-map prefetch) overlap the plan, which the kernel waits for on the device
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)ctx->num_sms);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, fixm, strm, lsem, a);
+    if (e != cudaSuccess) return cuda_fail(e, "tc kernel launch");
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "tc kernel launch");
 }
