@@ -452,17 +452,23 @@ def run_e2e(args, st, estp, dev, world):
         step()
     torch.cuda.synchronize()
     K = max(1, min(args.steps, 5))
-    if world > 1:
-        torch.distributed.barrier()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record()
-    for _ in range(K):
-        step()
-    b.record()
-    torch.cuda.synchronize()
+    # The host link is shared with other tenants of the machine, and single copies now and
+    # then run at a fraction of the link rate: time five blocks of K steps and report the
+    # median block (every block is listed).
+    blocks = []
+    for _ in range(5):
+        if world > 1:
+            torch.distributed.barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(K):
+            step()
+        b.record()
+        torch.cuda.synchronize()
+        ms, tokens = aggregate_ranks(a.elapsed_time(b), float(st.sumT), dev)
+        blocks.append(tokens * K / (ms / 1e3))
     st.ctx.sync_status()
-    ms, tokens = aggregate_ranks(a.elapsed_time(b), float(st.sumT), dev)
-    return {"value": tokens * K / (ms / 1e3), "unit": UNIT,
+    return {"value": sorted(blocks)[2], "unit": UNIT, "blocks": blocks,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": K,
             "pipeline": f"copy stream: Q/K/hidden, then logits in {n_chunks} row chunks; "
                         "attention after Q/K land, entropy per chunk as it lands"}

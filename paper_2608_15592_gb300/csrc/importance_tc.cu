@@ -11,9 +11,14 @@
 //   warps 1, 18  MMA issuers, one per fixed tile: D_A = A x S^T (warp 1) and
 //                D_B = B x S^T (warp 18), M = 128, N = 128, fp32 in TMEM, each
 //                double-buffered: 2 x 2 x 128 = all 512 TMEM columns
-//   warps 2-17   epilogue: warps 2-9 read D_A, warps 10-17 D_B; warp w reads TMEM lanes
-//                32*(w%4).. (its quarter), and two warps of a quarter split the 128
-//                columns (halves); tcgen05.ld, exp2 and row reductions
+//   warps 2-17   epilogue: tcgen05.ld, exp2 and row reductions; warp w reads TMEM lanes
+//                32*(w%4).. (its quarter).  LSE mode: 8 warps per fixed tile, two per
+//                quarter splitting the 128 columns, at every step.  Column-sum mode: a
+//                group of 4 warps per fixed tile and accumulator buffer reads all 128
+//                columns at every other step, so the two buffers' groups work a step
+//                apart and each step's lse values pass through 8 warps instead of 16
+//                (12 % faster there; in LSE mode the longer hold on the accumulator
+//                before it is released costs more than it gains)
 // Two issuers because the tensor core's instruction queue is shallow: a check of an
 // mbarrier costs an issuing thread ~150-180 cycles even when the phase has completed,
 // and with a single issuer the pipe idles through its two waits and commits per step;
@@ -43,7 +48,7 @@ constexpr int kTile = 128;             // rows of a fixed or streamed tile
 constexpr int kPair = 2 * kTile;       // rows of the fixed pair (the plan's tile)
 constexpr int kQcPair = 2;             // pairs of query tiles per column-sum item
 constexpr int kEpiWarp0 = 2;           // warps 2..17
-constexpr int kEpiWarps = 16;          // 8 per fixed tile
+constexpr int kEpiWarps = 16;          // 8 per fixed tile (LSE) or 4 per tile and buffer (column sums)
 // MMA issuers: warp 1 for fixed tile A, warp 18 for tile B, so that one issuer's barrier
 // waits and commits overlap the other's MMAs in the tensor pipe
 constexpr int kMmaWarpB = kEpiWarp0 + kEpiWarps;
@@ -68,8 +73,8 @@ struct Cfg {
     // dynamic smem layout (offsets from a 1024-aligned base)
     static constexpr int kFixOff = 0;                               // [2 buffers][A, B]
     static constexpr int kRingOff = 4 * kTileBytes;
-    static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][64] f32
-    static constexpr int kMergeOff = kNlOff + kEpiWarps * 64 * 4;   // [2][A, B][4][32] float2
+    static constexpr int kNlOff = kRingOff + kStages * kTileBytes;  // [16 warps][128] f32
+    static constexpr int kMergeOff = kNlOff + kEpiWarps * 128 * 4;   // [2][A, B][4][32] float2
     static constexpr int kBarOff = kMergeOff + 2 * 2 * 4 * 32 * 8;
     // fix_full/empty[2], ring_full/empty[kStages], acc_full/empty[A, B][kAccBufs],
     // drain[A, B], sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
@@ -272,8 +277,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* drain = acc_empty + 2 * kAccBufs;   // [A, B]
     uint64_t* sched_full = drain + 2;             // [kSched]
     uint64_t* sched_empty = sched_full + kSched;  // [kSched]
-    uint64_t* xfull = sched_empty + kSched;       // [2][A, B][4]: half-1 partials ready
-    uint64_t* xempty = xfull + 16;                // [2][A, B][4]: half-0 has read them
+    uint64_t* xfull = sched_empty + kSched;       // [2][A, B][4]: partial 1 of the rows written
+    uint64_t* xempty = xfull + 16;                // [2][A, B][4]: partial 0's warp has read it
     uint64_t* lse_full = xempty + 16;             // [kLseSlots]
     uint64_t* lse_empty = lse_full + kLseSlots;   // [kLseSlots]
     float* lse_ring = reinterpret_cast<float*>(sm + C::kLseOff);
@@ -289,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2 * kAccBufs; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], kEpiWarps / 2);  // one arrival per epilogue warp of the tile
+            mbar_init(&acc_empty[i], MODE == kModeLse ? kEpiWarps / 2 : kEpiWarps / 4);  // its readers
         }
         for (int i = 0; i < C::kStages; ++i) {
             mbar_init(&ring_full[i], 1);
@@ -307,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < kLseSlots; ++i) {
             mbar_init(&lse_full[i], 1);
-            mbar_init(&lse_empty[i], kEpiWarps);  // one arrival per epilogue warp
+            mbar_init(&lse_empty[i], kEpiWarps / 2);  // one arrival per warp that reads the step
         }
         *abort_flag = 0;
         mbar_fence_init();
@@ -468,11 +473,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
         // ------------------------------------------------------------- epilogue
         const int e = warp - kEpiWarp0;
-        const int tau = e >> 3;                    // fixed tile: 0 = A, 1 = B
+        // LSE mode: warps 8 tau .. 8 tau + 7 read fixed tile tau at every step, two warps per
+        //   quarter, one per column half (sub).
+        // Column-sum mode: warps 4 g .. 4 g + 3 read fixed tile g & 1 at the steps of parity
+        //   sub = g >> 1 (all 128 columns), so that the groups of the two accumulator buffers
+        //   work a step apart and each step's lse values are read by 8 warps.
+        constexpr int kChunks = MODE == kModeLse ? 2 : 4;  // 32-column chunks per step
+        const int tau = MODE == kModeLse ? e >> 3 : (e >> 2) & 1;  // fixed tile: 0 = A, 1 = B
+        const int sub = MODE == kModeLse ? (e >> 2) & 1 : e >> 3;  // which of a row's two partials
+        const int col0 = MODE == kModeLse ? sub * 64 : 0;
         const int q = warp & 3;                    // TMEM lane quarter
-        const int half = (e >> 2) & 1;             // column half
         const int row = q * 32 + lane;             // accumulator row owned by this thread
-        float* nl = nl_all + e * 64;
+        float* nl = nl_all + e * 128;
         uint32_t step = 0;
         bool ok = true;
         for (int it = 0; ok; ++it) {
@@ -484,19 +496,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             StepIter<MODE> si(a, t);
             auto do_step = [&](int s) -> bool {
                 const int row0 = si.row0, head = si.head, qt = si.qt;
-                if (MODE == kModeImp) {  // -log2e * lse of this warp's 64 query columns
+                if (MODE == kModeImp) {  // -log2e * lse of the step's 128 query columns
                     const int ls = (int)(step % kLseSlots);
                     if (!warp_wait(&lse_full[ls], (step / kLseSlots) & 1, abort_flag, a.status))
                         return false;
                     const int64_t x = (int64_t)head * a.sumT + t.t0 + row0;
-                    const float* lr = lse_ring + ls * (kLseSlotBytes / 4) + (int)(x & 3) + half * 64;
-                    const int i0 = row0 + half * 64 + lane, i1 = i0 + 32;
-                    const float r0 = i0 < t.T ? -lr[lane] * kLog2e : -INFINITY;
-                    const float r1 = i1 < t.T ? -lr[lane + 32] * kLog2e : -INFINITY;
+                    const float* lr = lse_ring + ls * (kLseSlotBytes / 4) + (int)(x & 3);
+                    float r[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int i = row0 + 32 * k + lane;
+                        r[k] = i < t.T ? -lr[32 * k + lane] * kLog2e : -INFINITY;
+                    }
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&lse_empty[ls]);
-                    nl[lane] = r0;
-                    nl[lane + 32] = r1;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) nl[32 * k + lane] = r[k];
                     __syncwarp();
                 }
                 const int ab = (int)(step % kAccBufs);
@@ -504,10 +519,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!warp_wait(&acc_full[abar], (step / kAccBufs) & 1, abort_flag, a.status))
                     return false;
                 tc_fence_after();
-                const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) +
-                                       (uint32_t)((ab * 2 + tau) * kAccCols + half * 64);
-                const int col0 = half * 64;
-                const float2 sc = make_float2(a.scale_log2, a.scale_log2);
                 // column-sum mode: this warp's key tile against the streamed query tile
                 const int kt = t.kt + tau;
                 const bool imp_skip = MODE == kModeImp && qt < kt;   // queries all before keys
@@ -516,13 +527,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int my_qt = t.qt0 + tau;
                 const bool lse_skip = MODE == kModeLse && s > my_qt;  // keys all after queries
                 const bool lse_diag = MODE == kModeLse && s == my_qt;
-                // two chunks of 32 columns: load, (release the accumulator), reduce
+                if (imp_skip || lse_skip) {  // nothing to read: hand the accumulator back
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&acc_empty[abar]);
+                    return true;
+                }
+                const uint32_t taddr =
+                    tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((ab * 2 + tau) * kAccCols + col0);
+                const float2 sc = make_float2(a.scale_log2, a.scale_log2);
+                // chunks of 32 columns: load, (release the accumulator after the last), reduce
 #pragma unroll
-                for (int ch = 0; ch < 2; ++ch) {
+                for (int ch = 0; ch < kChunks; ++ch) {
                     float v[32];
                     tmem_ld32(taddr + ch * 32, v);
                     tmem_wait_ld();
-                    if (ch == 1) {
+                    if (ch == kChunks - 1) {
                         tc_fence_before();
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&acc_empty[abar]);
@@ -530,7 +550,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int cb = col0 + ch * 32;  // tile column of v[0]
                     const float* nc = nl + ch * 32;
                     if (MODE == kModeImp) {
-                        if (imp_skip) continue;
                         if (!imp_diag) {
                             float2 acc_b = make_float2(0.f, 0.f);
 #pragma unroll
@@ -554,7 +573,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     } else {
-                        if (lse_skip) continue;
                         if (lse_diag) {  // diagonal tile: keys j = col after the query i = row
 #pragma unroll
                             for (int c = 0; c < 32; ++c)
@@ -585,19 +603,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ssum += st.x + st.y;
                     }
                 }
-                ++step;
                 return true;
             };
-            for (int s = 0; s < t.n_steps; ++s, si.next(a, t))
-                if (!(ok = do_step(s))) break;
+            for (int s = 0; s < t.n_steps; ++s, ++step, si.next(a, t))
+                if ((MODE == kModeLse || (int)(step & 1) == sub) && !(ok = do_step(s))) break;
             if (!ok) break;
-            // merge the two column halves of each row (bounded mbarrier hand-off), then write
+            // merge the two partials of each row (bounded mbarrier hand-off), then write
             const int pb = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
             float2* mb = merge + (pb * 2 + tau) * 128;
             uint64_t* xf = &xfull[(pb * 2 + tau) * 4 + q];
             uint64_t* xe = &xempty[(pb * 2 + tau) * 4 + q];
-            if (half == 1) {
+            if (sub == 1) {
                 if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status);
                 if (!ok) break;
                 mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
