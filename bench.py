@@ -199,9 +199,7 @@ class Step:
         self.pooled = torch.empty(w.B, w.D, dtype=torch.float32, device=device)
         self.pred = torch.empty(w.B, dtype=torch.float32, device=device)
         self.ctx = estp.Context(torch.cuda.current_device())
-        n_layers = len(w.layers)
-        # launches per step: entropy 2; per layer lse 2 + importance 3; finalize 1; pool 2
-        self.launches = 2 + n_layers * 5 + 1 + 2
+        self.launches = st_launches(w)
 
     def run(self, ev=None):
         """One step on the current stream; ev: dict of (start, end) events per kernel."""
@@ -393,7 +391,10 @@ def st_tokens(w):
 
 
 def st_launches(w):
-    return 2 + len(w.layers) * 5 + 1 + 4
+    """Library launches per step: entropy 2 (kernel + merge); per layer, the row
+    normaliser 2 (plan + kernel) and the column sums 3 (plan + kernel + reduce); the
+    finalize 1; pooling 2 (stream + finish)."""
+    return 2 + len(w.layers) * 5 + 1 + 2
 
 
 def run_e2e(args, st, estp, dev, world):

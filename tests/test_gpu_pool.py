@@ -137,3 +137,40 @@ def test_pool_bad_cu_then_good(cuda_lib):
     P_ref = oracle.pool(hid, H.astype(np.float64), S.astype(np.float64), cu, 0.7, 0.3, 1.0)
     assert_pooled(pooled.cpu().numpy(), P_ref)
     assert_pred(pred.cpu().numpy(), oracle.length_head(P_ref, Wt, b, c))
+
+
+def test_pool_deterministic_and_counters(cuda_lib):
+    """Fixed-order merges: repeated calls give identical bits. The head's per-prompt
+    arrival counters are back to zero after every call: a head-less call with several
+    column slices, calls with the head, then a call of another shape on the same
+    context, all exact."""
+    cu, hid, H, S, hd = _inputs(synth.BF16, [2000, 7, 0, 300, 1], 8192)
+    Wt, b, c = _head(32, 8192)
+    head = cuda_lib.Head(torch.from_numpy(Wt).cuda(), torch.from_numpy(b).cuda(),
+                         torch.from_numpy(c).cuda())
+    ctx = cuda_lib.Context(0)
+    Hd, Sd, cud = (torch.from_numpy(H).cuda(), torch.from_numpy(S).cuda(),
+                   torch.as_tensor(cu, device="cuda"))
+    P_ref = oracle.pool(hid, H.astype(np.float64), S.astype(np.float64), cu, 0.7, 0.3, 1.0)
+    pooled0, _ = ctx.pool(hd, Hd, Sd, cud, 0.7, 0.3, 1.0)
+    ctx.sync_status()
+    assert_pooled(pooled0.cpu().numpy(), P_ref)
+    runs = []
+    for _ in range(3):
+        pooled, pred = ctx.pool(hd, Hd, Sd, cud, 0.7, 0.3, 1.0, head=head)
+        ctx.sync_status()
+        runs.append((pooled.cpu().numpy(), pred.cpu().numpy()))
+    for p, y in runs[1:]:
+        assert np.array_equal(p, runs[0][0]) and np.array_equal(y, runs[0][1])
+    assert np.array_equal(runs[0][0], pooled0.cpu().numpy())
+    assert_pred(runs[0][1], oracle.length_head(P_ref, Wt, b, c))
+    cu2, hid2, H2, S2, hd2 = _inputs(synth.BF16, [50, 0, 700], 1024, seed=8)
+    Wt2, b2, c2 = _head(32, 1024)
+    head2 = cuda_lib.Head(torch.from_numpy(Wt2).cuda(), torch.from_numpy(b2).cuda(),
+                          torch.from_numpy(c2).cuda())
+    pooled2, pred2 = ctx.pool(hd2, torch.from_numpy(H2).cuda(), torch.from_numpy(S2).cuda(),
+                              torch.as_tensor(cu2, device="cuda"), 0.7, 0.3, 1.0, head=head2)
+    ctx.sync_status()
+    P2 = oracle.pool(hid2, H2.astype(np.float64), S2.astype(np.float64), cu2, 0.7, 0.3, 1.0)
+    assert_pooled(pooled2.cpu().numpy(), P2)
+    assert_pred(pred2.cpu().numpy(), oracle.length_head(P2, Wt2, b2, c2))
