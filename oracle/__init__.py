@@ -6,6 +6,7 @@ reference arm may import this package.  It wraps ``liboracle.so`` (plain C in
 
 Functions and the paper passages they follow (arXiv 2608.15592):
   token_entropy   Eq. 2-1 (Sec. 3.2)
+  lm_head_entropy Eq. 2-1 of the logits h W^T formed from hidden states
   attn_lse        the row normaliser of the causal softmax A (Sec. 3.1)
   attn_colsum     sum_i A_ij of Eq. 2-0 for one layer, summed over query heads
   attn_colsum_rows  the same from the rows i >= row_from only (exact for late keys)
@@ -53,6 +54,7 @@ class _Lib:
         P, I, I64, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
         sig = {
             "oracle_token_entropy": [P, I, I64, I64, I64, P, I],
+            "oracle_lm_head_entropy": [P, P, I, I64, I64, I64, I64, I64, P, I],
             "oracle_attn_lse": [P, P, I, I, I, I, D, P, I, P, I],
             "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
             "oracle_attn_colsum_rows": [P, P, I, I, I, I, D, P, I, P, I, I, I64, P, I],
@@ -147,6 +149,20 @@ def token_entropy(logits: np.ndarray, V: int | None = None, n_threads: int = 0) 
     out = np.zeros(rows, dtype=np.float64)
     _check(_load().oracle_token_entropy(_ptr(logits), _dtype_code(logits), rows, V, ld,
                                         _ptr(out), n_threads), "token_entropy")
+    return out
+
+
+def lm_head_entropy(hidden: np.ndarray, W: np.ndarray, n_threads: int = 0) -> np.ndarray:
+    """Eq. 2-1 per row of hidden [rows, D] with the logits hidden @ W^T, W [V, D] (same
+    element type; bf16 as raw uint16 bits)."""
+    hidden, W = np.ascontiguousarray(hidden), np.ascontiguousarray(W)
+    assert hidden.dtype == W.dtype and hidden.ndim == 2 and W.ndim == 2
+    rows, D = hidden.shape
+    V, Dw = W.shape
+    assert Dw == D
+    out = np.zeros(rows, dtype=np.float64)
+    _check(_load().oracle_lm_head_entropy(_ptr(hidden), _ptr(W), _dtype_code(hidden), rows, D,
+                                          V, D, D, _ptr(out), n_threads), "lm_head_entropy")
     return out
 
 

@@ -123,6 +123,55 @@ int oracle_token_entropy(const void* logits, int dtype, int64_t n_rows, int64_t 
     return 0;
 }
 
+/* ------------------------------- Eq. 2-1 with the logits formed in place */
+
+typedef struct {
+    const void *hid, *W;
+    int dtype;
+    int64_t D, V, ldh, ldw;
+    double* H;
+} lm_head_ctx;
+
+/* One row: the logits z_v = sum_k h_k W_vk of the output projection (W holds one row
+ * of D weights per vocabulary entry), formed in double, then Eq. 2-1 of z exactly as
+ * in entropy_unit.  scratch: [D + V] doubles. */
+static void lm_head_entropy_unit(void* vctx, int64_t r, double* scratch) {
+    lm_head_ctx* c = (lm_head_ctx*)vctx;
+    double* h = scratch;
+    double* z = scratch + c->D;
+    for (int64_t k = 0; k < c->D; ++k) h[k] = load_elem(c->hid, c->dtype, r * c->ldh + k);
+    for (int64_t v = 0; v < c->V; ++v) {
+        double dot = 0.0;
+        for (int64_t k = 0; k < c->D; ++k) dot += h[k] * load_elem(c->W, c->dtype, v * c->ldw + k);
+        z[v] = dot;
+    }
+    double m = -INFINITY;
+    for (int64_t v = 0; v < c->V; ++v)
+        if (z[v] > m) m = z[v];
+    double s = 0.0;
+    for (int64_t v = 0; v < c->V; ++v) {
+        z[v] = exp(z[v] - m);
+        s += z[v];
+    }
+    double H = 0.0;
+    for (int64_t v = 0; v < c->V; ++v) {
+        double p = z[v] / s;
+        if (p > 0.0) H += -p * log(p);
+    }
+    c->H[r] = H;
+}
+
+int oracle_lm_head_entropy(const void* hidden, const void* W, int dtype, int64_t n_rows,
+                           int64_t D, int64_t V, int64_t ldh, int64_t ldw, double* H_out,
+                           int n_threads) {
+    if (!valid_dtype(dtype) || n_rows < 0 || D <= 0 || V <= 0 || ldh < D || ldw < D) return -1;
+    if (n_rows == 0) return 0;
+    if (!hidden || !W || !H_out) return -1;
+    lm_head_ctx c = {hidden, W, dtype, D, V, ldh, ldw, H_out};
+    parallel_units(lm_head_entropy_unit, &c, n_rows, (size_t)(D + V), n_threads);
+    return 0;
+}
+
 /* ------------------------------------------- attention rows (Sec. 3.1) */
 
 /* One (prompt, query head) pair: the prompt's q^h and k^{h/rep} rows widened to

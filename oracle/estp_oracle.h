@@ -10,6 +10,7 @@
  * "When Entropy Is Not Enough: Reclaiming Lost Semantics in LLM Output Length
  * Prediction"), evaluated in IEEE double precision:
  *   oracle_token_entropy       Eq. 2-1  (Sec. 3.2)
+ *   oracle_lm_head_entropy     Eq. 2-1 of the logits h W^T of the output projection
  *   oracle_attn_lse            log-normaliser of the softmax rows of A (Sec. 3.1)
  *   oracle_attn_colsum         the column sums of A inside Eq. 2-0 (Sec. 3.1)
  *   oracle_importance          Eq. 2-0 (the 1/N scaling and the head/layer mean)
@@ -41,6 +42,14 @@ enum { ORACLE_F32 = 0, ORACLE_BF16 = 1 };
  * logits: n_rows rows of V values, row stride ld elements.  H_out: [n_rows]. */
 int oracle_token_entropy(const void* logits, int dtype, int64_t n_rows, int64_t V,
                          int64_t ld, double* H_out, int n_threads);
+
+/* Eq. 2-1 of logits that are formed here from hidden states: z_rv = sum_k h_rk W_vk
+ * (the model's output projection; W: V rows of D weights, row stride ldw), then
+ * H_r = -sum_v p_rv ln p_rv with p_r = softmax(z_r).  hidden: n_rows rows of D values,
+ * row stride ldh.  H_out: [n_rows]. */
+int oracle_lm_head_entropy(const void* hidden, const void* W, int dtype, int64_t n_rows,
+                           int64_t D, int64_t V, int64_t ldh, int64_t ldw, double* H_out,
+                           int n_threads);
 
 /* Row log-normaliser of causal attention for one layer:
  * lse_out[h * sumT + i] = ln sum_{j <= i, j in prompt(i)} exp(scale * q_i^h . k_j^{h/rep}).

@@ -91,6 +91,61 @@ def pin_entropy_shift_perm_pad():
 
 # ------------------------------------------------------- Eq. 2-0 importance
 
+def pin_lm_head_zero_weights():
+    """Logits formed from hidden states: W = 0 gives uniform logits, H = ln V."""
+    rng = _rng(41)
+    for V, D in ((1, 8), (7, 3), (300, 64)):
+        h = rng.standard_normal((3, D)).astype(np.float32)
+        W = np.zeros((V, D), dtype=np.float32)
+        _close(oracle.lm_head_entropy(h, W), [math.log(V)] * 3, what="W = 0")
+
+
+def pin_lm_head_two_level():
+    """A hidden row c e_k reads column k of W only: with a entries x / c and V - a zeros
+    there, the logits are two-level (a at x, V - a at 0) and H has the closed form of the
+    two-level pin, whatever the other columns of W hold."""
+    rng = _rng(42)
+    for V, D, a, x, k in ((50, 6, 3, 2.5, 4), (1000, 16, 999, -1.25, 0), (64, 3, 1, 0.5, 2)):
+        c = 2.0
+        W = rng.standard_normal((V, D)).astype(np.float64)
+        W[:, k] = 0.0
+        W[rng.choice(V, a, replace=False), k] = x / c
+        h = np.zeros((1, D))
+        h[0, k] = c
+        Z = a * math.exp(x) + V - a
+        p, q = math.exp(x) / Z, 1.0 / Z
+        ref = -a * p * math.log(p) - (V - a) * q * math.log(q)
+        _close(oracle.lm_head_entropy(h.astype(np.float32), W.astype(np.float32)), [ref],
+               rtol=1e-6, what="two-level from hidden")
+
+
+def pin_lm_head_bruteforce():
+    """Tiny shapes, fp32 and bf16: a pure-Python triple loop forms every logit and the
+    entropy with math.exp / math.log."""
+    from synth import bf16_bits_to_f32
+    rng = _rng(43)
+    for rows, D, V in ((3, 5, 7), (2, 9, 1), (4, 1, 11)):
+        h = rng.standard_normal((rows, D)).astype(np.float32) * 2
+        W = rng.standard_normal((V, D)).astype(np.float32)
+        for bf16 in (False, True):
+            if bf16:
+                hb, Wb = (np.asarray(x).view(np.uint32) >> 16 for x in (h, W))
+                hb, Wb = hb.astype(np.uint16), Wb.astype(np.uint16)
+                hv, Wv = bf16_bits_to_f32(hb).astype(np.float64), bf16_bits_to_f32(Wb).astype(np.float64)
+                got = oracle.lm_head_entropy(hb, Wb)
+            else:
+                hv, Wv = h.astype(np.float64), W.astype(np.float64)
+                got = oracle.lm_head_entropy(h, W)
+            ref = []
+            for r in range(rows):
+                z = [sum(float(hv[r, k]) * float(Wv[v, k]) for k in range(D)) for v in range(V)]
+                m = max(z)
+                e = [math.exp(t - m) for t in z]
+                sm = sum(e)
+                ref.append(-sum((x / sm) * math.log(x / sm) for x in e if x > 0))
+            _close(got, ref, rtol=1e-12, atol=1e-12, what=f"brute force bf16={bf16}")
+
+
 def _brute_colsum(Q, K, cu, scale, heads=None, exclude_self=False):
     """Full masked score matrix per (prompt, head); rows via scipy softmax."""
     Qd = Q.astype(np.float64) if Q.dtype != np.uint16 else _bf(Q)

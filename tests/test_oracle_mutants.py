@@ -15,6 +15,11 @@ MUTANTS = [
     ("entropy unnormalised", "double p = e[v] / s;", "double p = e[v];"),
     ("entropy ignores row stride", "int64_t off = r * c->ld;", "int64_t off = r * c->V;"),
     ("bf16 widening shift", "[idx] << 16;", "[idx] << 15;"),
+    ("lm-head dot drops the last coordinate",
+     "for (int64_t k = 0; k < c->D; ++k) dot +=", "for (int64_t k = 0; k < c->D - 1; ++k) dot +="),
+    ("lm-head W transposed", "load_elem(c->W, c->dtype, v * c->ldw + k)",
+     "load_elem(c->W, c->dtype, k * c->V + v)"),
+    ("lm-head entropy sign", "H += -p * log(p);", "H += p * log(p);"),
     ("scores unscaled", "s[j] = c->scale * dot;", "s[j] = dot;"),
     ("row sums instead of column sums", "col[j] += exp(s[j] - m) / Z;",
      "col[i] += exp(s[j] - m) / Z;"),
