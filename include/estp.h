@@ -109,6 +109,27 @@ estp_status estp_token_entropy_noalloc(const void* logits, estp_dtype dtype, int
                                        int64_t V, int64_t ld, float* entropy_out,
                                        estp_stream_t stream);
 
+/* Token entropy with the logits formed on the GPU and never stored: Eq. 2-1 (Sec. 3.2)
+ * of z_r = h_r W^T, where h_r is token r's final hidden state and W the model's output
+ * projection (the LM head).  For a model with a large vocabulary the logits are the
+ * largest tensor of the feature path; here they live only in tensor memory, one
+ * 128 x 256 tile at a time.
+ *   hidden      : bf16 [n_rows, ldh] row-major (first D columns used), 16-byte aligned
+ *   ldh         : row stride in elements, >= D and a multiple of 8
+ *   W           : bf16 [V, ldw] row-major: one row of D weights per vocabulary entry
+ *                 (the usual lm_head.weight layout), 16-byte aligned
+ *   ldw         : row stride in elements, >= D and a multiple of 8
+ *   dtype       : ESTP_BF16 (anything else is ESTP_ERR_UNSUPPORTED)
+ *   D           : hidden size, a positive multiple of 64
+ *   V           : vocabulary size >= 1
+ *   entropy_out : fp32 [n_rows], natural log
+ * The products accumulate in fp32 on the tensor cores; the entropy is formed in fp32 from
+ * the fp32 logits.  n_rows = 0 is a no-op.  Uses the context's workspace (12 bytes per row
+ * and vocabulary split).  Repeated calls give identical bits. */
+estp_status estp_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ldh, const void* W,
+                                 int64_t ldw, estp_dtype dtype, int64_t n_rows, int64_t D,
+                                 int64_t V, float* entropy_out, estp_stream_t stream);
+
 /* ------------------------------------------------------------------ (b)
  * Attention layout for one layer (Sec. 3.1): Q is [sumT, Hq, head_dim] and K is
  * [sumT, Hkv, head_dim], row-major and contiguous, dtype ESTP_BF16 or ESTP_F32.

@@ -36,7 +36,7 @@ _DIVISOR_FLAGS = {"length": 0, "causal": ESTP_IMP_DIV_CAUSAL, "none": ESTP_IMP_D
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
            "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
-           "estp_head_loss", "estp_misalignment")
+           "estp_head_loss", "estp_misalignment", "estp_lm_head_entropy")
 
 
 class EstpError(RuntimeError):
@@ -80,6 +80,8 @@ def _load():
         "estp_head_loss": ([P, P, I32, I64, ctypes.POINTER(_Head), P, F, P, P, P, P, P],
                            ctypes.c_int),
         "estp_misalignment": ([P, P, P, P, I32, I64, I32, P, P], ctypes.c_int),
+        "estp_lm_head_entropy": ([P, P, I64, P, I64, ctypes.c_int, I64, I64, I64, P, P],
+                                 ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -148,6 +150,23 @@ class Context:
         _check(lib.estp_sync_status(self._h, _stream(stream)))
 
     # ------------------------------------------------------------------ (a)
+    def lm_head_entropy(self, hidden, W, out=None, stream=None):
+        """estp_lm_head_entropy: entropy (nats) of softmax(hidden @ W^T) per row, the logits
+        formed on the tensor cores and never stored.  hidden: bf16 [rows, D], W: bf16 [V, D]
+        (row views of wider arrays allowed: stride(1) == 1)."""
+        import torch
+        assert hidden.dim() == 2 and W.dim() == 2 and hidden.shape[1] == W.shape[1]
+        assert hidden.numel() == 0 or hidden.stride(1) == 1
+        assert W.stride(1) == 1
+        rows, D = hidden.shape
+        V = W.shape[0]
+        ldh = hidden.stride(0) if rows > 1 else D
+        ldw = W.stride(0) if V > 1 else D
+        out = torch.empty(rows, dtype=torch.float32, device=hidden.device) if out is None else out
+        _check(lib.estp_lm_head_entropy(self._h, _ptr(hidden), ldh, _ptr(W), ldw, _dtype(hidden),
+                                        rows, D, V, _ptr(out), _stream(stream)))
+        return out
+
     def token_entropy(self, logits, V: int | None = None, cu_seqlens=None, out=None,
                       stream=None):
         """estp_token_entropy on a 2-D [rows, ld] tensor (stride(1) == 1)."""

@@ -311,6 +311,26 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
                             grad_bias, grad_pooled, reinterpret_cast<cudaStream_t>(stream));
 }
 
+estp_status estp_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ldh, const void* W,
+                                 int64_t ldw, estp_dtype dtype, int64_t n_rows, int64_t D,
+                                 int64_t V, float* entropy_out, estp_stream_t stream) {
+    if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
+    if (dtype != ESTP_BF16) return fail(ESTP_ERR_UNSUPPORTED, "lm-head entropy: bf16 only");
+    if (n_rows < 0 || D < 64 || D % 64 || V < 1)
+        return fail(ESTP_ERR_INVALID_ARG, "need n_rows >= 0, D a positive multiple of 64, V >= 1");
+    if (ldh < D || ldw < D || ldh % 8 || ldw % 8)
+        return fail(ESTP_ERR_INVALID_ARG, "need ldh, ldw >= D and multiples of 8");
+    if (n_rows > INT32_MAX || V > INT32_MAX) return fail(ESTP_ERR_INVALID_ARG, "n_rows, V < 2^31");
+    if (n_rows == 0) return ESTP_OK;
+    if (!hidden || !W || !entropy_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    if (!aligned16(hidden) || !aligned16(W))
+        return fail(ESTP_ERR_INVALID_ARG, "hidden and W must be 16-byte aligned");
+    estp_status st = set_device(ctx);
+    if (st != ESTP_OK) return st;
+    return launch_lm_head_entropy(ctx, hidden, ldh, W, ldw, n_rows, D, V, entropy_out,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
+
 estp_status estp_misalignment(estp_ctx* ctx, const float* entropy, const float* importance,
                               const int32_t* cu_seqlens, int32_t B, int64_t sumT, int32_t pct,
                               int32_t* counts_out, estp_stream_t stream) {
