@@ -309,6 +309,7 @@ def run_ours(args, rank, world, local_rank):
     e2e = run_e2e(args, st, estp, dev, world)
     head_loss = time_head_loss(st, dev)
     misalign = time_misalignment(st)
+    lm_head = time_lm_head(st, bf16_sus)
     clocks = clk.summary()
     del st
     if rank != 0:
@@ -326,7 +327,7 @@ def run_ours(args, rank, world, local_rank):
                    "l2": "inputs larger than L2 (~6.4 GB per step), no flush"},
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": st_launches(w) * K, "clocks": clocks,
-        "head_loss": head_loss, "misalignment": misalign,
+        "head_loss": head_loss, "misalignment": misalign, "lm_head_entropy": lm_head,
     }
 
 
@@ -355,6 +356,41 @@ def time_head_loss(st, dev, iters: int = 50):
     nbytes = 4 * (2 * K * D + 2 * B * D + K * D + K + B * D + B * K)
     return {"ms": ms, "B": B, "D": D, "K": K, "launches": 2, "bytes": nbytes,
             "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "launch"}
+
+
+def time_lm_head(st, peak_tflops, iters: int = 20, warmup: int = 30):
+    """Token entropy with the logits formed from the step's hidden states and a seeded
+    output projection W [V, D] (estp_lm_head_entropy): not part of the step, which
+    reads materialised logits; timed on its own with CUDA events. Algorithmic work is
+    2 sumT D V flops of the projection; the logits it does not write and read back are
+    2 sumT V bytes. A call runs for many milliseconds at full tensor rate, so the GPU
+    settles under its power cap: ~0.4 s of warm-up calls come first, and the figure is
+    compared with the sustained bf16 peak."""
+    import numpy as np
+    import torch
+    import synth
+    from synth import device as sd
+    w = st.w
+    W = sd.normal(synth.stream_key(w.seed, 101), (w.V, w.D), synth.BF16, scale=3.0 / np.sqrt(w.D))
+    H = torch.empty(st.sumT, dtype=torch.float32, device=W.device)
+    for _ in range(warmup):
+        st.ctx.lm_head_entropy(st.hidden, W, out=H)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        st.ctx.lm_head_entropy(st.hidden, W, out=H)
+    b.record()
+    torch.cuda.synchronize()
+    st.ctx.sync_status()
+    ms = a.elapsed_time(b) / iters
+    flops = 2.0 * st.sumT * w.D * w.V
+    tf = flops / (ms / 1e3) / 1e12
+    del W
+    return {"ms": ms, "rows": st.sumT, "D": w.D, "V": w.V, "flops": flops, "launches": 2,
+            "bound": "tensor", "achieved": tf, "unit": "TFLOP/s", "peak": peak_tflops,
+            "frac": tf / peak_tflops, "tokens_per_s": st.sumT / (ms / 1e3),
+            "logit_bytes_not_stored": 2 * st.sumT * w.V}
 
 
 def time_misalignment(st, iters: int = 50):

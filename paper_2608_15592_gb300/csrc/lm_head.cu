@@ -408,10 +408,28 @@ estp_status launch_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ld
     a.nk = (int)(D / kKc);
     a.n_vt = (int)((V + kN - 1) / kN);
     const int64_t n_rb = (n_rows + kM - 1) / kM;
-    // splits: about eight items per SM (a short last wave), at most one tile per split
-    int64_t S = (8 * (int64_t)ctx->num_sms + n_rb - 1) / n_rb;
-    if (S > a.n_vt) S = a.n_vt;
-    if (S < 1) S = 1;
+    // splits: at least four items per SM; the fewest splits whose items fill the last
+    // wave of the persistent grid to 97 % (else the best fill up to four times as many).
+    // Fewer splits keep more row blocks in flight at once, so that each W tile read from
+    // DRAM serves more of them.
+    // At least as many splits that the row blocks in flight at once (G / S of them, 256 D
+    // bytes each) fit in ~48 MB of L2 beside the W tiles streaming through.
+    const int64_t G = ctx->num_sms;
+    const int64_t l2_budget = 48ll << 20, rb_bytes = (int64_t)kM * D * 2;
+    const int64_t s_l2 = (G * rb_bytes + l2_budget - 1) / l2_budget;
+    int64_t s_lo = (4 * G + n_rb - 1) / n_rb;
+    if (s_lo < s_l2) s_lo = s_l2;
+    int64_t S = s_lo < a.n_vt ? s_lo : a.n_vt;  // small problems: one tile per split
+    double best = -1.0;
+    for (int64_t c = s_lo; c <= a.n_vt && c <= 4 * s_lo; ++c) {
+        const int64_t items = n_rb * c, waves = (items + G - 1) / G;
+        const double fill = (double)items / (double)(waves * G);
+        if (fill > best + 1e-9) {
+            best = fill;
+            S = c;
+        }
+        if (fill >= 0.97) break;
+    }
     a.S = (int)S;
     a.n_items = n_rb * S;
     s = ws_reserve(ctx, sizeof(float) * 3 * (size_t)S * (size_t)n_rows);

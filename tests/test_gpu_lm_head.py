@@ -66,11 +66,14 @@ def test_lm_head_entropy_strided_rows(cuda_lib):
     assert np.abs(H.cpu().numpy() - _ref(h, W)).max() <= TOL
 
 
-def test_lm_head_entropy_qwen_shape(cuda_lib):
-    """The 16-prompt batch's output projection: hidden size 3584, vocabulary 152064, 2000
-    tokens (16 row blocks, the last ragged); sampled rows against the oracle, which forms
-    each row's 152064 logits in double.  Two calls give identical bits."""
-    rows, D, V = 2000, 3584, 152064
+@pytest.mark.parametrize("rows", [2000, 21663])
+def test_lm_head_entropy_qwen_shape(cuda_lib, rows):
+    """The output projection of the 16-prompt batch: hidden size 3584, vocabulary 152064,
+    2000 tokens (76 vocabulary splits) and the batch's 21663 tokens (170 row blocks, 8
+    splits, the launch the bench times), the last row block ragged; sampled rows against
+    the oracle, which forms each row's 152064 logits in double.  Two calls give identical
+    bits."""
+    D, V = 3584, 152064
     h, W = _inputs(rows, D, V, 3.0, seed=13)
     ctx = cuda_lib.Context(0)
     H = ctx.lm_head_entropy(h, W)
@@ -78,7 +81,7 @@ def test_lm_head_entropy_qwen_shape(cuda_lib):
     ctx.sync_status()
     Hn = H.cpu().numpy()
     assert np.array_equal(Hn, H2.cpu().numpy())
-    pick = np.asarray([0, 1, 127, 128, 1023, 1920, 1998, 1999])
+    pick = np.unique(np.asarray([0, 1, 127, 128, 1023, 1920, rows // 2, rows - 129, rows - 2, rows - 1]))
     ref = _ref(h, W, pick)
     err = np.abs(Hn[pick].astype(np.float64) - ref)
     assert err.max() <= TOL, f"max err {err.max():.2e} at rows {pick[np.argmax(err)]}"
