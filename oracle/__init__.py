@@ -14,6 +14,8 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   pool            Eqs. 2-2, 2-3, 2-4
   length_head     Eq. 3-2 with a linear projection
   head_loss       Eqs. 3-1, 3-3 (soft-label CE + MSE) and their gradients
+  mlp_length_head Eq. 3-2 behind the one-hidden-layer ReLU MLP predictor
+  mlp_head_loss   Eqs. 3-1, 3-3 through that MLP, and every gradient
   misalignment    the entropy/importance misalignment counts of Sec. 1 (Fig. 1b), numpy
 
 bf16 arrays are passed as numpy uint16 holding the raw bfloat16 bits.
@@ -63,6 +65,8 @@ class _Lib:
             "oracle_pool": [P, I, I64, I64, P, P, P, I, D, D, D, P, P],
             "oracle_length_head": [P, I, I64, P, P, P, I, P, P],
             "oracle_head_loss": [P, I, I64, P, P, P, I, P, D, P, P, P, P],
+            "oracle_mlp_length_head": [P, I, I64, P, P, I, P, P, P, I, P, P],
+            "oracle_mlp_head_loss": [P, I, I64, P, P, I, P, P, P, I, P, D, P, P, P, P, P, P],
         }
         for name, args in sig.items():
             fn = getattr(lib, name)
@@ -282,6 +286,45 @@ def head_loss(pooled, W, bias, centers, y, lambda3: float, grads: bool = True):
                                     _ptr(y), float(lambda3), _ptr(loss), _ptr(gW), _ptr(gb),
                                     _ptr(gp)), "head_loss")
     return (float(loss[0]), gW, gb, gp) if grads else float(loss[0])
+
+
+def _mlp_args(W1, b1, W2, b2, centers):
+    W1 = np.ascontiguousarray(W1, dtype=np.float32)
+    W2 = np.ascontiguousarray(W2, dtype=np.float32)
+    b1 = None if b1 is None else np.ascontiguousarray(b1, dtype=np.float32)
+    b2 = None if b2 is None else np.ascontiguousarray(b2, dtype=np.float32)
+    return W1, b1, W2, b2, np.ascontiguousarray(centers, dtype=np.float32)
+
+
+def mlp_length_head(pooled, W1, b1, W2, b2, centers, return_probs: bool = False):
+    """Eq. 3-2 behind the MLP u = relu(W1 h + b1), z = W2 u + b2: y_hat [B] (and p_hat)."""
+    pooled = np.ascontiguousarray(pooled, dtype=np.float64)
+    B, D = pooled.shape
+    W1, b1, W2, b2, centers = _mlp_args(W1, b1, W2, b2, centers)
+    F, K = W1.shape[0], W2.shape[0]
+    y = np.zeros(B)
+    p = np.zeros((B, K)) if return_probs else None
+    _check(_load().oracle_mlp_length_head(_ptr(pooled), B, D, _ptr(W1), _ptr(b1), F, _ptr(W2),
+                                          _ptr(b2), _ptr(centers), K, _ptr(p), _ptr(y)),
+           "mlp_length_head")
+    return (y, p) if return_probs else y
+
+
+def mlp_head_loss(pooled, W1, b1, W2, b2, centers, y, lambda3: float, grads: bool = True):
+    """Eqs. 3-1, 3-3 through the MLP predictor; returns the loss and, if asked,
+    (grad_W1 [F, D], grad_b1 [F], grad_W2 [K, F], grad_b2 [K], grad_pooled [B, D])."""
+    pooled = np.ascontiguousarray(pooled, dtype=np.float64)
+    B, D = pooled.shape
+    W1, b1, W2, b2, centers = _mlp_args(W1, b1, W2, b2, centers)
+    F, K = W1.shape[0], W2.shape[0]
+    y = np.ascontiguousarray(y, dtype=np.float32)
+    loss = np.zeros(1)
+    g = [np.zeros((F, D)), np.zeros(F), np.zeros((K, F)), np.zeros(K), np.zeros((B, D))] if grads \
+        else [None] * 5
+    _check(_load().oracle_mlp_head_loss(_ptr(pooled), B, D, _ptr(W1), _ptr(b1), F, _ptr(W2),
+                                        _ptr(b2), _ptr(centers), K, _ptr(y), float(lambda3),
+                                        _ptr(loss), *[_ptr(x) for x in g]), "mlp_head_loss")
+    return (float(loss[0]), *g) if grads else float(loss[0])
 
 
 def misalignment(H, S, cu_seqlens, pct: int = 40) -> np.ndarray:

@@ -458,3 +458,76 @@ int oracle_head_loss(const double* pooled, int B, int64_t D, const float* W, con
     free(ph); free(yh); free(dz);
     return 0;
 }
+
+
+/* ---------------------------------------- the MLP predictor (Sec. 3.3, Fig. 2) */
+
+/* Hidden layer of the MLP head: a_bf = sum_x W1_fx h_bx + b1_f, u_bf = max(a_bf, 0).
+ * Returns a [B, F] array of u (caller frees), or NULL. */
+static double* mlp_hidden(const double* pooled, int B, int64_t D, const float* W1, const float* b1,
+                          int F) {
+    double* u = (double*)malloc(sizeof(double) * (size_t)B * F);
+    if (!u) return NULL;
+    for (int b = 0; b < B; ++b)
+        for (int f = 0; f < F; ++f) {
+            double a = b1 ? (double)b1[f] : 0.0;
+            for (int64_t x = 0; x < D; ++x) a += (double)W1[(int64_t)f * D + x] * pooled[(int64_t)b * D + x];
+            u[(int64_t)b * F + f] = a > 0.0 ? a : 0.0;
+        }
+    return u;
+}
+
+int oracle_mlp_length_head(const double* pooled, int B, int64_t D, const float* W1, const float* b1,
+                           int F, const float* W2, const float* b2, const float* centers, int K,
+                           double* probs_out, double* y_out) {
+    if (B <= 0 || D <= 0 || F <= 0 || !pooled || !W1 || !W2) return -1;
+    double* u = mlp_hidden(pooled, B, D, W1, b1, F);
+    if (!u) return -1;
+    const int r = oracle_length_head(u, B, F, W2, b2, centers, K, probs_out, y_out);
+    free(u);
+    return r;
+}
+
+/* The loss of Eq. 3-3 through the MLP: the second layer is the linear head of Eq. 3-2 on u,
+ * whose loss and gradients (dL/dW2, dL/db2, dL/du) come from oracle_head_loss; the chain
+ * rule then goes through the ReLU (dL/da = dL/du where a > 0, else 0) and the first
+ * layer: dL/dW1_fx = sum_b dL/da_bf h_bx, dL/db1_f = sum_b dL/da_bf,
+ * dL/dh_bx = sum_f W1_fx dL/da_bf. */
+int oracle_mlp_head_loss(const double* pooled, int B, int64_t D, const float* W1, const float* b1,
+                         int F, const float* W2, const float* b2, const float* centers, int K,
+                         const float* y, double lambda3, double* loss_out, double* grad_W1,
+                         double* grad_b1, double* grad_W2, double* grad_b2, double* grad_pooled) {
+    if (B <= 0 || D <= 0 || F <= 0 || !pooled || !W1 || !W2) return -1;
+    double* u = mlp_hidden(pooled, B, D, W1, b1, F);
+    double* du = (double*)malloc(sizeof(double) * (size_t)B * F);
+    if (!u || !du) { free(u); free(du); return -1; }
+    if (oracle_head_loss(u, B, F, W2, b2, centers, K, y, lambda3, loss_out, grad_W2, grad_b2, du) != 0) {
+        free(u); free(du);
+        return -1;
+    }
+    for (int64_t q = 0; q < (int64_t)B * F; ++q)
+        if (!(u[q] > 0.0)) du[q] = 0.0;  /* dL/da: the ReLU passes the gradient where a > 0 */
+    if (grad_W1)
+        for (int f = 0; f < F; ++f)
+            for (int64_t x = 0; x < D; ++x) {
+                double g = 0.0;
+                for (int b = 0; b < B; ++b) g += du[(int64_t)b * F + f] * pooled[(int64_t)b * D + x];
+                grad_W1[(int64_t)f * D + x] = g;
+            }
+    if (grad_b1)
+        for (int f = 0; f < F; ++f) {
+            double g = 0.0;
+            for (int b = 0; b < B; ++b) g += du[(int64_t)b * F + f];
+            grad_b1[f] = g;
+        }
+    if (grad_pooled)
+        for (int b = 0; b < B; ++b)
+            for (int64_t x = 0; x < D; ++x) {
+                double g = 0.0;
+                for (int f = 0; f < F; ++f) g += (double)W1[(int64_t)f * D + x] * du[(int64_t)b * F + f];
+                grad_pooled[(int64_t)b * D + x] = g;
+            }
+    free(u);
+    free(du);
+    return 0;
+}

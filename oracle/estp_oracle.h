@@ -18,6 +18,8 @@
  *   oracle_pool                Eqs. 2-2, 2-3, 2-4 (Sec. 3.2)
  *   oracle_length_head         Eq. 3-2 (Sec. 3.3), linear projection + softmax
  *   oracle_head_loss           Eqs. 3-1 and 3-3 (Sec. 3.3) and their gradients
+ *   oracle_mlp_length_head     Eq. 3-2 behind a one-hidden-layer ReLU MLP (Sec. 3.3, Fig. 2)
+ *   oracle_mlp_head_loss       Eqs. 3-1 and 3-3 through that MLP, and every gradient
  *
  * Parity status: every function is pinned by the CPU tests (closed forms,
  * invariants, brute force against independent library routines); none is
@@ -116,6 +118,23 @@ int oracle_length_head(const double* pooled, int B, int64_t D, const float* W,
 int oracle_head_loss(const double* pooled, int B, int64_t D, const float* W, const float* bias,
                      const float* centers, int K, const float* y, double lambda3,
                      double* loss_out, double* grad_W, double* grad_bias, double* grad_pooled);
+
+/* The MLP predictor of Sec. 3.3 (Fig. 2 names an MLP; its depth, width and activation are
+ * not given, read here as one hidden layer of F ReLU units):
+ *   u_b = max(W1 h_b + b1, 0),  z_b = W2 u_b + b2,  p_hat_b = softmax(z_b),
+ *   y_hat_b = sum_k p_hat_bk c_k.
+ * W1: [F, D] fp32, b1: [F] or NULL, W2: [K, F] fp32, b2: [K] or NULL.
+ * oracle_mlp_length_head writes y_out [B] and, if probs_out != NULL, p_hat [B, K].
+ * oracle_mlp_head_loss writes the loss of Eq. 3-3 (batch mean, as oracle_head_loss) and
+ * each gradient whose pointer is not NULL: grad_W1 [F, D], grad_b1 [F], grad_W2 [K, F],
+ * grad_b2 [K], grad_pooled [B, D].  The ReLU's derivative at a = 0 is taken as 0. */
+int oracle_mlp_length_head(const double* pooled, int B, int64_t D, const float* W1, const float* b1,
+                           int F, const float* W2, const float* b2, const float* centers, int K,
+                           double* probs_out, double* y_out);
+int oracle_mlp_head_loss(const double* pooled, int B, int64_t D, const float* W1, const float* b1,
+                         int F, const float* W2, const float* b2, const float* centers, int K,
+                         const float* y, double lambda3, double* loss_out, double* grad_W1,
+                         double* grad_b1, double* grad_W2, double* grad_b2, double* grad_pooled);
 
 #ifdef __cplusplus
 }

@@ -571,4 +571,97 @@ def pin_misalignment():
     assert abs(big[0, 1] / big[0, 0] - 0.4) < 0.02 and abs(big[0, 2] / big[0, 0] - 0.4) < 0.02
 
 
+def _mlp_case(rng, B, D, F, K, spread=1.0):
+    h = rng.standard_normal((B, D))
+    W1 = (rng.standard_normal((F, D)) / np.sqrt(D)).astype(np.float32)
+    b1 = (rng.standard_normal(F) * 0.5).astype(np.float32)
+    W2 = (rng.standard_normal((K, F)) * spread / np.sqrt(F)).astype(np.float32)
+    b2 = rng.standard_normal(K).astype(np.float32)
+    c = ((np.arange(K) + 0.5) * 16.0).astype(np.float32)
+    y = rng.uniform(0, 16.0 * K, B).astype(np.float32)
+    return h, W1, b1, W2, b2, c, y
+
+
+def pin_mlp_reduces_to_linear():
+    """With F = D, W1 = I and b1 = 50 every hidden unit is active and u = h + 50, so the
+    MLP predictor is the linear head of Eq. 3-2 on h + 50: the same y_hat, loss, dL/dW2,
+    dL/db2, and dL/dh = dL/du; dL/dW1 and dL/db1 are the outer products of dL/du with h
+    and its batch sum."""
+    rng = _rng(51)
+    B, D, K = 4, 6, 9
+    h = rng.standard_normal((B, D))
+    W2 = rng.standard_normal((K, D)).astype(np.float32)
+    b2 = rng.standard_normal(K).astype(np.float32)
+    c = ((np.arange(K) + 0.5) * 10.0).astype(np.float32)
+    y = rng.uniform(0, 90, B).astype(np.float32)
+    W1, b1 = np.eye(D, dtype=np.float32), np.full(D, 50.0, dtype=np.float32)
+    u = h + 50.0
+    _close(oracle.mlp_length_head(h, W1, b1, W2, b2, c), oracle.length_head(u, W2, b2, c),
+           rtol=1e-12, what="MLP y_hat vs linear head")
+    for lam in (0.0, 0.3, 1.0):
+        L, gW1, gb1, gW2, gb2, gh = oracle.mlp_head_loss(h, W1, b1, W2, b2, c, y, lam)
+        Ll, gW, gb, gu = oracle.head_loss(u, W2, b2, c, y, lam)
+        _close([L], [Ll], rtol=1e-12, what="MLP loss vs linear")
+        _close(gW2, gW, rtol=1e-12, atol=1e-12, what="dL/dW2")
+        _close(gb2, gb, rtol=1e-12, atol=1e-12, what="dL/db2")
+        _close(gh, gu, rtol=1e-12, atol=1e-12, what="dL/dh")
+        _close(gb1, gu.sum(0), rtol=1e-12, atol=1e-12, what="dL/db1")
+        _close(gW1, gu.T @ h, rtol=1e-10, atol=1e-12, what="dL/dW1")
+
+
+def pin_mlp_dead_units():
+    """W1 = 0 and b1 < 0 switch every hidden unit off: u = 0, so z = b2 for every prompt,
+    y_hat = sum softmax(b2)_k c_k (scipy), the loss is the linear head's on zero features,
+    and no gradient reaches W1, b1 or h."""
+    rng = _rng(52)
+    B, D, F, K = 3, 7, 5, 8
+    h = rng.standard_normal((B, D))
+    W1, b1 = np.zeros((F, D), np.float32), np.full(F, -1.0, np.float32)
+    W2 = rng.standard_normal((K, F)).astype(np.float32)
+    b2 = rng.standard_normal(K).astype(np.float32)
+    c = ((np.arange(K) + 0.5) * 10.0).astype(np.float32)
+    y = rng.uniform(0, 80, B).astype(np.float32)
+    ref = float(np.dot(special.softmax(b2.astype(np.float64)), c.astype(np.float64)))
+    _close(oracle.mlp_length_head(h, W1, b1, W2, b2, c), [ref] * B, rtol=1e-12, what="dead y_hat")
+    L, gW1, gb1, gW2, gb2, gh = oracle.mlp_head_loss(h, W1, b1, W2, b2, c, y, 0.4)
+    _close([L], [oracle.head_loss(np.zeros((B, F)), W2, b2, c, y, 0.4, grads=False)], rtol=1e-12,
+           what="dead loss")
+    assert not np.any(gW1) and not np.any(gb1) and not np.any(gh), "gradient through dead units"
+    assert not np.any(gW2), "dL/dW2 = dz^T u = 0"
+
+
+def pin_mlp_finite_differences():
+    """Every gradient of the MLP loss equals central differences of the loss (units kept
+    away from the ReLU's kink)."""
+    rng = _rng(53)
+    B, D, F, K = 3, 5, 4, 6
+    for _ in range(20):
+        h, W1, b1, W2, b2, c, y = _mlp_case(rng, B, D, F, K, spread=2.0)
+        a = h @ W1.T.astype(np.float64) + b1
+        if np.min(np.abs(a)) > 0.05:
+            break
+    lam = 0.35
+    L, gW1, gb1, gW2, gb2, gh = oracle.mlp_head_loss(h, W1, b1, W2, b2, c, y, lam)
+    loss = lambda hh, w1, bb1, w2, bb2: oracle.mlp_head_loss(hh, w1, bb1, w2, bb2, c, y, lam, grads=False)
+
+    def fd(arr, grad, call, eps):
+        arr64 = np.array(arr, dtype=np.float64)
+        num = np.zeros(arr64.shape)
+        for idx in np.ndindex(arr64.shape):
+            up, dn = arr64.copy(), arr64.copy()
+            up[idx] += eps
+            dn[idx] -= eps
+            num[idx] = (call(up) - call(dn)) / (2 * eps)
+        scale = max(np.max(np.abs(num)), 1e-12)
+        assert np.max(np.abs(num - grad)) <= 1e-3 * scale, f"finite differences: {np.max(np.abs(num - grad))}"
+
+    # W1, b1, W2, b2 are fp32 arguments of the oracle: steps of 2^-10 keep them exact
+    eps = 1.0 / 1024
+    fd(h, gh, lambda v: loss(v, W1, b1, W2, b2), 1e-5)
+    fd(W1, gW1, lambda v: loss(h, v.astype(np.float32), b1, W2, b2), eps)
+    fd(b1, gb1, lambda v: loss(h, W1, v.astype(np.float32), W2, b2), eps)
+    fd(W2, gW2, lambda v: loss(h, W1, b1, v.astype(np.float32), b2), eps)
+    fd(b2, gb2, lambda v: loss(h, W1, b1, W2, v.astype(np.float32)), eps)
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

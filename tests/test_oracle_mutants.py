@@ -58,6 +58,14 @@ MUTANTS = [
      "((double)centers[k] - yh[b]));"),
     ("feature gradient through W transposed", "g += (double)wk[x] * dz[k];",
      "g += (double)W[x * K + k] * dz[k];"),
+    ("MLP without its ReLU", "u[(int64_t)b * F + f] = a > 0.0 ? a : 0.0;",
+     "u[(int64_t)b * F + f] = a;"),
+    ("MLP first layer transposed", "(double)W1[(int64_t)f * D + x] * pooled",
+     "(double)W1[(int64_t)x * F + f] * pooled"),
+    ("MLP gradient passes switched-off units", "if (!(u[q] > 0.0)) du[q] = 0.0;", ""),
+    ("MLP input gradient through W1 transposed", "(double)W1[(int64_t)f * D + x] * du",
+     "(double)W1[(int64_t)x * F + f] * du"),
+    ("MLP first-layer bias gradient averaged", "grad_b1[f] = g;", "grad_b1[f] = g / (double)B;"),
 ]
 
 
