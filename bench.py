@@ -354,8 +354,30 @@ def time_head_loss(st, dev, iters: int = 50):
     st.ctx.sync_status()
     ms = a.elapsed_time(b) / iters
     nbytes = 4 * (2 * K * D + 2 * B * D + K * D + K + B * D + B * K)
-    return {"ms": ms, "B": B, "D": D, "K": K, "launches": 2, "bytes": nbytes,
-            "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "launch"}
+    out = {"ms": ms, "B": B, "D": D, "K": K, "launches": 2, "bytes": nbytes,
+           "achieved_gbs": nbytes / (ms / 1e3) / 1e9, "bound": "launch"}
+    # the MLP predictor (one ReLU layer of F = 1024 units), its loss and all gradients
+    import paper_2608_15592_gb300 as estp
+    F = 1024
+    W1 = torch.randn(F, D, generator=g, device=dev) / D ** 0.5
+    b1 = torch.randn(F, generator=g, device=dev) * 0.3
+    W2 = torch.randn(K, F, generator=g, device=dev) * (3.0 / F ** 0.5)
+    mlp = estp.MlpHead(W1, b1, W2, st.head.bias, st.head.centers)
+    for _ in range(3):
+        st.ctx.mlp_head_loss(st.pooled, mlp, targets, 0.5)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(iters):
+        st.ctx.mlp_head_loss(st.pooled, mlp, targets, 0.5)
+    b.record()
+    torch.cuda.synchronize()
+    st.ctx.sync_status()
+    ms = a.elapsed_time(b) / iters
+    # W1 read by the hidden layer and by both of its gradients, dL/dW1 written
+    mbytes = 4 * (3 * F * D + F * D + 2 * K * F + 4 * B * D + 4 * B * F)
+    out["mlp"] = {"ms": ms, "F": F, "launches": 4, "bytes": mbytes,
+                  "achieved_gbs": mbytes / (ms / 1e3) / 1e9, "bound": "launch / L2"}
+    return out
 
 
 def time_lm_head(st, peak_tflops, iters: int = 20, warmup: int = 30):

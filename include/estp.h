@@ -245,6 +245,50 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
                            float* loss_out, float* grad_W, float* grad_bias,
                            float* grad_pooled, estp_stream_t stream);
 
+/* The MLP predictor of Sec. 3.3 (Fig. 2 feeds the pooled representation to "an MLP
+ * predictor"; its depth, width and activation are not given, and are read here as one
+ * hidden layer of F ReLU units in front of the K-bin softmax projection of Eq. 3-2):
+ *   u_b = max(W1 h_b + b1, 0),  z_b = W2 u_b + b2,  p_hat_b = softmax(z_b),
+ *   y_hat_b = sum_k p_hat_bk c_k.
+ * All arrays fp32, caller-owned device memory; the struct itself is a HOST pointer. */
+typedef struct {
+    const float* W1;       /* [F, D] */
+    const float* b1;       /* [F] or NULL */
+    const float* W2;       /* [K, F] */
+    const float* b2;       /* [K] or NULL */
+    const float* centers;  /* [K] bin centres c_k */
+    int32_t F;             /* hidden units, >= 1 */
+    int32_t K;             /* bins, 1..1024 */
+} estp_mlp_head;
+
+/* Gradients of estp_mlp_head_loss; every pointer may be NULL (not computed). */
+typedef struct {
+    float* W1;      /* [F, D] */
+    float* b1;      /* [F] */
+    float* W2;      /* [K, F] */
+    float* b2;      /* [K] */
+    float* pooled;  /* [B, D] */
+} estp_mlp_grads;
+
+/* Predicted lengths through the MLP predictor: pred_out [B] = y_hat_b, and, when
+ * probs_out is not NULL, probs_out [B, K] = p_hat_b.  pooled: fp32 [B, D] (estp_pool's
+ * pooled_out).  B >= 1, D >= 1. */
+estp_status estp_mlp_head_predict(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                                  const estp_mlp_head* head, float* pred_out, float* probs_out,
+                                  estp_stream_t stream);
+
+/* The loss of Eq. 3-3 (soft labels of Eq. 3-1 around the bin nearest to y_b, ties to the
+ * lower bin; batch mean, as estp_head_loss) through the MLP predictor, and its gradients:
+ * the second layer as the linear head on u, then the chain rule through the ReLU (its
+ * derivative at 0 taken as 0) and the first layer.
+ *   targets  : fp32 [B] target lengths y_b;  lambda3: weight of the cross-entropy term
+ *   loss_out : fp32 [1];  grads: HOST pointer, or NULL for the loss alone
+ * Every sum runs in a fixed order (no atomics), so repeated calls give identical bits. */
+estp_status estp_mlp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                               const estp_mlp_head* head, const float* targets, float lambda3,
+                               float* loss_out, const estp_mlp_grads* grads,
+                               estp_stream_t stream);
+
 /* Entropy/importance misalignment, the diagnostic behind Fig. 1b and Sec. 3.1's
  * motivation (not part of the predictor).  Per prompt b, with k = floor(pct*T_b/100),
  * TopX and BotX are the k tokens with the largest and with the smallest X (ties: the

@@ -36,7 +36,8 @@ _DIVISOR_FLAGS = {"length": 0, "causal": ESTP_IMP_DIV_CAUSAL, "none": ESTP_IMP_D
 EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
            "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
-           "estp_head_loss", "estp_misalignment", "estp_lm_head_entropy")
+           "estp_head_loss", "estp_misalignment", "estp_lm_head_entropy",
+           "estp_mlp_head_predict", "estp_mlp_head_loss")
 
 
 class EstpError(RuntimeError):
@@ -54,6 +55,17 @@ class MixParams(ctypes.Structure):
 class _Head(ctypes.Structure):
     _fields_ = [("W", ctypes.c_void_p), ("bias", ctypes.c_void_p),
                 ("centers", ctypes.c_void_p), ("K", ctypes.c_int32)]
+
+
+class _MlpHead(ctypes.Structure):
+    _fields_ = [("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("W2", ctypes.c_void_p),
+                ("b2", ctypes.c_void_p), ("centers", ctypes.c_void_p), ("F", ctypes.c_int32),
+                ("K", ctypes.c_int32)]
+
+
+class _MlpGrads(ctypes.Structure):
+    _fields_ = [("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("W2", ctypes.c_void_p),
+                ("b2", ctypes.c_void_p), ("pooled", ctypes.c_void_p)]
 
 
 def _load():
@@ -80,6 +92,10 @@ def _load():
         "estp_head_loss": ([P, P, I32, I64, ctypes.POINTER(_Head), P, F, P, P, P, P, P],
                            ctypes.c_int),
         "estp_misalignment": ([P, P, P, P, I32, I64, I32, P, P], ctypes.c_int),
+        "estp_mlp_head_predict": ([P, P, I32, I64, ctypes.POINTER(_MlpHead), P, P, P],
+                                  ctypes.c_int),
+        "estp_mlp_head_loss": ([P, P, I32, I64, ctypes.POINTER(_MlpHead), P, F, P,
+                                ctypes.POINTER(_MlpGrads), P], ctypes.c_int),
         "estp_lm_head_entropy": ([P, P, I64, P, I64, ctypes.c_int, I64, I64, I64, P, P],
                                  ctypes.c_int),
     }
@@ -122,6 +138,17 @@ class Head:
     """Linear length head (Eq. 3-2): W [K, D], bias [K] or None, centers [K], fp32 CUDA."""
     W: "object"
     bias: "object"
+    centers: "object"
+
+
+@dataclass
+class MlpHead:
+    """MLP predictor (Sec. 3.3): u = relu(W1 h + b1), z = W2 u + b2, then Eq. 3-2.
+    W1 [F, D], b1 [F] or None, W2 [K, F], b2 [K] or None, centers [K], fp32 CUDA."""
+    W1: "object"
+    b1: "object"
+    W2: "object"
+    b2: "object"
     centers: "object"
 
 
@@ -253,6 +280,42 @@ class Context:
         _check(lib.estp_head_loss(self._h, _ptr(pooled), B, D, hp, _ptr(targets), lambda3,
                                   _ptr(loss), _ptr(gW), _ptr(gb), _ptr(gp), _stream(stream)))
         return (loss, gW, gb, gp) if grads else loss
+
+    @staticmethod
+    def _mlp(head: "MlpHead"):
+        return ctypes.pointer(_MlpHead(_ptr(head.W1), _ptr(head.b1), _ptr(head.W2), _ptr(head.b2),
+                                       _ptr(head.centers), head.W1.shape[0], head.W2.shape[0]))
+
+    def mlp_head_predict(self, pooled, head: "MlpHead", probs: bool = False, stream=None):
+        """estp_mlp_head_predict: predicted lengths [B] (and p_hat [B, K] if probs)."""
+        import torch
+        B, D = pooled.shape
+        pred = torch.empty(B, dtype=torch.float32, device=pooled.device)
+        p = torch.empty(B, head.W2.shape[0], dtype=torch.float32, device=pooled.device) if probs else None
+        _check(lib.estp_mlp_head_predict(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(pred),
+                                         _ptr(p), _stream(stream)))
+        return (pred, p) if probs else pred
+
+    def mlp_head_loss(self, pooled, head: "MlpHead", targets, lambda3: float, grads=True,
+                      stream=None):
+        """estp_mlp_head_loss (Eqs. 3-1, 3-3 through the MLP predictor): returns loss [1]
+        and, if grads, (dL/dW1 [F, D], dL/db1 [F], dL/dW2 [K, F], dL/db2 [K], dL/dpooled
+        [B, D]).  grads may also be a set of those names to compute only some of them."""
+        import torch
+        B, D = pooled.shape
+        F, K = head.W1.shape[0], head.W2.shape[0]
+        dev = pooled.device
+        shapes = {"W1": (F, D), "b1": (F,), "W2": (K, F), "b2": (K,), "pooled": (B, D)}
+        want = set(shapes) if grads is True else (set(grads) if grads else set())
+        out = {k: torch.empty(v, dtype=torch.float32, device=dev) if k in want else None
+               for k, v in shapes.items()}
+        loss = torch.empty(1, dtype=torch.float32, device=dev)
+        gp = ctypes.pointer(_MlpGrads(*[_ptr(out[k]) for k in ("W1", "b1", "W2", "b2", "pooled")]))
+        _check(lib.estp_mlp_head_loss(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(targets),
+                                      lambda3, _ptr(loss), gp if want else None, _stream(stream)))
+        if not grads:
+            return loss
+        return (loss, *[out[k] for k in ("W1", "b1", "W2", "b2", "pooled")])
 
     def pool(self, hidden, entropy, importance, cu_seqlens, lambda1: float, lambda2: float,
              alpha: float, head: Head | None = None, D: int | None = None, pooled=None,

@@ -331,6 +331,44 @@ estp_status estp_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ldh,
                                   reinterpret_cast<cudaStream_t>(stream));
 }
 
+static estp_status check_mlp(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                             const estp_mlp_head* head) {
+    if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
+    if (B < 1 || D < 1) return fail(ESTP_ERR_INVALID_ARG, "need B >= 1 and D >= 1");
+    if (!head || !head->W1 || !head->W2 || !head->centers || head->F < 1 || head->K < 1 ||
+        head->K > 1024)
+        return fail(ESTP_ERR_INVALID_ARG, "MLP head needs W1, W2, centers, F >= 1, 1 <= K <= 1024");
+    if (!pooled) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    return ESTP_OK;
+}
+
+estp_status estp_mlp_head_predict(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                                  const estp_mlp_head* head, float* pred_out, float* probs_out,
+                                  estp_stream_t stream) {
+    estp_status st = check_mlp(ctx, pooled, B, D, head);
+    if (st != ESTP_OK) return st;
+    if (!pred_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    st = set_device(ctx);
+    if (st != ESTP_OK) return st;
+    return launch_mlp_head_predict(ctx, pooled, B, D, *head, pred_out, probs_out,
+                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+estp_status estp_mlp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
+                               const estp_mlp_head* head, const float* targets, float lambda3,
+                               float* loss_out, const estp_mlp_grads* grads,
+                               estp_stream_t stream) {
+    estp_status st = check_mlp(ctx, pooled, B, D, head);
+    if (st != ESTP_OK) return st;
+    if (!std::isfinite(lambda3)) return fail(ESTP_ERR_INVALID_ARG, "lambda3 must be finite");
+    if (!targets || !loss_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
+    st = set_device(ctx);
+    if (st != ESTP_OK) return st;
+    const estp_mlp_grads none = {nullptr, nullptr, nullptr, nullptr, nullptr};
+    return launch_mlp_head_loss(ctx, pooled, B, D, *head, targets, lambda3, loss_out,
+                                grads ? *grads : none, reinterpret_cast<cudaStream_t>(stream));
+}
+
 estp_status estp_misalignment(estp_ctx* ctx, const float* entropy, const float* importance,
                               const int32_t* cu_seqlens, int32_t B, int64_t sumT, int32_t pct,
                               int32_t* counts_out, estp_stream_t stream) {

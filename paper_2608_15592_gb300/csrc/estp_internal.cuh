@@ -108,6 +108,12 @@ estp_status launch_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t 
 estp_status launch_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ldh, const void* W,
                                    int64_t ldw, int64_t n_rows, int64_t D, int64_t V, float* H,
                                    cudaStream_t st);
+estp_status launch_mlp_head_predict(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                                    const estp_mlp_head& head, float* pred, float* probs,
+                                    cudaStream_t st);
+estp_status launch_mlp_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                                 const estp_mlp_head& head, const float* targets, float lambda3,
+                                 float* loss, const estp_mlp_grads& g, cudaStream_t st);
 estp_status launch_misalignment(estp_ctx* ctx, const float* H, const float* S, const int32_t* cu,
                                 int B, int64_t sumT, int pct, int32_t* counts, cudaStream_t st);
 estp_status launch_importance_finalize(estp_ctx* ctx, const float* acc, const int32_t* cu, int B,

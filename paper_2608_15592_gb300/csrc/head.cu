@@ -1,5 +1,7 @@
 // Training loss of the length head (Sec. 3.3): the soft label of Eq. 3-1, the linear
-// head of Eq. 3-2 and the loss of Eq. 3-3 averaged over the prompts, with its gradients.
+// head of Eq. 3-2 and the loss of Eq. 3-3 averaged over the prompts, with its gradients;
+// and the MLP predictor of Sec. 3.3 / Fig. 2 (one hidden layer of F ReLU units in front
+// of the K-bin softmax projection), its prediction and its loss.
 //
 // head_fwd_kernel: CTA b forms z = W h_b + bias (warp w takes logits k = w, w + 8, ...:
 //   lanes stride the D columns, then a fixed butterfly), p_hat = softmax(z),
@@ -9,6 +11,11 @@
 // head_grad_kernel: one thread per output element of dL/dW = sum_b dz_b h_b^T,
 //   dL/dbias = sum_b dz_b and dL/dpooled_b = W^T dz_b, each summed in a fixed order,
 //   and the loss itself.  Everything is fp32.
+// mlp_hidden_kernel: u = max(W1 h + b1, 0), one warp per hidden unit and 8 prompts at a
+//   time (lanes stride D, then a fixed butterfly).  The MLP reuses the two kernels above
+//   layer by layer: head_fwd_kernel and head_grad_kernel on u with W2 (dL/dW2, dL/db2,
+//   dL/du and the loss), then head_grad_kernel on h with W1, gated by u > 0 (the ReLU's
+//   derivative), for dL/dW1, dL/db1 and dL/dh.
 #include "estp_internal.cuh"
 
 namespace estp {
@@ -27,7 +34,7 @@ __global__ void __launch_bounds__(kFwdThreads) head_fwd_kernel(
     const float* __restrict__ pooled, int64_t D, const float* __restrict__ W,
     const float* __restrict__ bias, const float* __restrict__ centers, int K,
     const float* __restrict__ targets, int B, float lambda3, float* __restrict__ dz,
-    float2* __restrict__ part) {
+    float2* __restrict__ part, float* __restrict__ pred, float* __restrict__ probs) {
     __shared__ float z_s[kMaxK];
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
@@ -45,7 +52,6 @@ __global__ void __launch_bounds__(kFwdThreads) head_fwd_kernel(
     // y_hat is formed relative to the centre of the largest logit r: y_hat = c_r + dy with
     // dy = sum_k p_hat_k (c_k - c_r), so that c_k - y_hat = (c_k - c_r) - dy does not
     // cancel when p_hat is concentrated on r.
-    const float y = targets[b];
     float m = -INFINITY;
     int r = 0;
     for (int k = lane; k < K; k += 32)
@@ -58,18 +64,25 @@ __global__ void __launch_bounds__(kFwdThreads) head_fwd_kernel(
     }
     const float cr = centers[r];
     float Z = 0.f, dy = 0.f;
-    float best_d = INFINITY;
-    int best_k = 0;
     for (int k = lane; k < K; k += 32) {
         const float e = __expf(z_s[k] - m);
         Z += e;
         dy = fmaf(e, centers[k] - cr, dy);
-        const float d = fabsf(y - centers[k]);
-        if (d < best_d) { best_d = d; best_k = k; }  // lowest k of this lane on a tie
     }
     Z = warp_sum(Z);
     dy = warp_sum(dy) / Z;
     const float yh = cr + dy;
+    if (pred && lane == 0) pred[b] = yh;
+    if (probs)
+        for (int k = lane; k < K; k += 32) probs[(int64_t)b * K + k] = __expf(z_s[k] - m) / Z;
+    if (!targets) return;  // prediction only
+    const float y = targets[b];
+    float best_d = INFINITY;
+    int best_k = 0;
+    for (int k = lane; k < K; k += 32) {
+        const float d = fabsf(y - centers[k]);
+        if (d < best_d) { best_d = d; best_k = k; }  // lowest k of this lane on a tie
+    }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {  // (distance, index): the lowest index wins ties
         const float od = __shfl_xor_sync(0xffffffffu, best_d, off);
@@ -94,35 +107,41 @@ __global__ void __launch_bounds__(kFwdThreads) head_fwd_kernel(
     if (lane == 0) part[b] = make_float2(ce, err * err);
 }
 
+// gate (NULL: none): dz[b, k] counts only where gate[b, k] > 0 (a ReLU's derivative);
+// loss NULL: no loss element.
 __global__ void head_grad_kernel(const float* __restrict__ pooled, int B, int64_t D,
                                  const float* __restrict__ W, int K, const float* __restrict__ dz,
-                                 const float2* __restrict__ part, float lambda3,
-                                 float* __restrict__ loss, float* __restrict__ grad_W,
+                                 const float* __restrict__ gate, const float2* __restrict__ part,
+                                 float lambda3, float* __restrict__ loss, float* __restrict__ grad_W,
                                  float* __restrict__ grad_bias, float* __restrict__ grad_pooled) {
     const int64_t n_w = grad_W ? (int64_t)K * D : 0;
     const int64_t n_b = grad_bias ? K : 0;
     const int64_t n_p = grad_pooled ? (int64_t)B * D : 0;
-    const int64_t total = n_w + n_b + n_p + 1;
+    const int64_t total = n_w + n_b + n_p + (loss ? 1 : 0);
+    auto dzg = [&](int b, int k) -> float {
+        const float v = dz[(int64_t)b * K + k];
+        return gate && !(gate[(int64_t)b * K + k] > 0.f) ? 0.f : v;
+    };
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
          t += (int64_t)gridDim.x * blockDim.x) {
         if (t < n_w) {  // dL/dW[k, x] = sum_b dz[b, k] h[b, x]
             const int k = (int)(t / D);
             const int64_t x = t - (int64_t)k * D;
-            float g = 0.f;
-            for (int b = 0; b < B; ++b) g = fmaf(dz[(int64_t)b * K + k], pooled[(int64_t)b * D + x], g);
-            grad_W[t] = g;
+            float acc = 0.f;
+            for (int b = 0; b < B; ++b) acc = fmaf(dzg(b, k), pooled[(int64_t)b * D + x], acc);
+            grad_W[t] = acc;
         } else if (t < n_w + n_b) {  // dL/dbias[k] = sum_b dz[b, k]
             const int k = (int)(t - n_w);
-            float g = 0.f;
-            for (int b = 0; b < B; ++b) g += dz[(int64_t)b * K + k];
-            grad_bias[k] = g;
+            float acc = 0.f;
+            for (int b = 0; b < B; ++b) acc += dzg(b, k);
+            grad_bias[k] = acc;
         } else if (t < n_w + n_b + n_p) {  // dL/dpooled[b, x] = sum_k W[k, x] dz[b, k]
             const int64_t r = t - n_w - n_b;
             const int b = (int)(r / D);
             const int64_t x = r - (int64_t)b * D;
-            float g = 0.f;
-            for (int k = 0; k < K; ++k) g = fmaf(W[(int64_t)k * D + x], dz[(int64_t)b * K + k], g);
-            grad_pooled[r] = g;
+            float acc = 0.f;
+            for (int k = 0; k < K; ++k) acc = fmaf(W[(int64_t)k * D + x], dzg(b, k), acc);
+            grad_pooled[r] = acc;
         } else {  // the loss: batch means of the CE and squared-error terms
             float ce = 0.f, se = 0.f;
             for (int b = 0; b < B; ++b) {
@@ -132,6 +151,44 @@ __global__ void head_grad_kernel(const float* __restrict__ pooled, int B, int64_
             loss[0] = (lambda3 * ce + (1.f - lambda3) * se) / (float)B;
         }
     }
+}
+
+constexpr int kHidB = 8;  // prompts per warp pass of the hidden layer
+
+// u[b, f] = max(sum_x W1[f, x] h[b, x] + b1[f], 0): warp w of the grid takes hidden
+// unit f = w, and the prompts kHidB at a time.
+__global__ void __launch_bounds__(256) mlp_hidden_kernel(const float* __restrict__ pooled,
+                                                         int B, int64_t D,
+                                                         const float* __restrict__ W1,
+                                                         const float* __restrict__ b1, int F,
+                                                         float* __restrict__ u) {
+    const int lane = threadIdx.x & 31;
+    const int64_t f = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (f >= F) return;
+    const float* w = W1 + f * D;
+    const float bias = b1 ? b1[f] : 0.f;
+    for (int b0 = 0; b0 < B; b0 += kHidB) {
+        const int nb = B - b0 < kHidB ? B - b0 : kHidB;
+        float acc[kHidB];
+#pragma unroll
+        for (int j = 0; j < kHidB; ++j) acc[j] = 0.f;
+        for (int64_t x = lane; x < D; x += 32) {
+            const float wx = w[x];
+#pragma unroll
+            for (int j = 0; j < kHidB; ++j)
+                if (j < nb) acc[j] = fmaf(wx, pooled[(int64_t)(b0 + j) * D + x], acc[j]);
+        }
+#pragma unroll
+        for (int j = 0; j < kHidB; ++j) {
+            const float a = warp_sum(acc[j]) + bias;
+            if (lane == 0 && j < nb) u[(int64_t)(b0 + j) * F + f] = a > 0.f ? a : 0.f;
+        }
+    }
+}
+
+int grad_blocks(estp_ctx* ctx, int64_t total) {
+    const int64_t b = (total + 255) / 256, cap = 4 * (int64_t)ctx->num_sms;
+    return (int)(b < cap ? (b > 0 ? b : 1) : cap);
 }
 
 }  // namespace
@@ -148,15 +205,72 @@ estp_status launch_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t 
     float* dz = reinterpret_cast<float*>(ws);
     float2* part = reinterpret_cast<float2*>(ws + off_part);
     head_fwd_kernel<<<B, kFwdThreads, 0, st>>>(pooled, D, head.W, head.bias, head.centers, K,
-                                               targets, B, lambda3, dz, part);
+                                               targets, B, lambda3, dz, part, nullptr, nullptr);
     const int64_t total = (grad_W ? (int64_t)K * D : 0) + (grad_bias ? K : 0) +
                           (grad_pooled ? (int64_t)B * D : 0) + 1;
-    const int blocks = (int)((total + 255) / 256 < 4 * (int64_t)ctx->num_sms ? (total + 255) / 256
-                                                                           : 4 * (int64_t)ctx->num_sms);
-    head_grad_kernel<<<blocks, 256, 0, st>>>(pooled, B, D, head.W, K, dz, part, lambda3, loss,
-                                             grad_W, grad_bias, grad_pooled);
+    head_grad_kernel<<<grad_blocks(ctx, total), 256, 0, st>>>(pooled, B, D, head.W, K, dz, nullptr,
+                                                              part, lambda3, loss, grad_W, grad_bias,
+                                                              grad_pooled);
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "head loss launch");
+}
+
+// The MLP's hidden units u [B, F] into the workspace at `u`.
+static cudaError_t mlp_hidden(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                              const estp_mlp_head& head, float* u, cudaStream_t st) {
+    const int64_t threads = 32 * (int64_t)head.F;
+    mlp_hidden_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(pooled, B, D, head.W1,
+                                                                        head.b1, head.F, u);
+    return cudaGetLastError();
+}
+
+estp_status launch_mlp_head_predict(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                                    const estp_mlp_head& head, float* pred, float* probs,
+                                    cudaStream_t st) {
+    estp_status s = ws_reserve(ctx, sizeof(float) * (size_t)B * head.F);
+    if (s != ESTP_OK) return s;
+    float* u = static_cast<float*>(ctx->ws);
+    cudaError_t e = mlp_hidden(ctx, pooled, B, D, head, u, st);
+    if (e != cudaSuccess) return cuda_fail(e, "mlp hidden launch");
+    head_fwd_kernel<<<B, kFwdThreads, 0, st>>>(u, head.F, head.W2, head.b2, head.centers, head.K,
+                                               nullptr, B, 0.f, nullptr, nullptr, pred, probs);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "mlp head launch");
+}
+
+estp_status launch_mlp_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t D,
+                                 const estp_mlp_head& head, const float* targets, float lambda3,
+                                 float* loss, const estp_mlp_grads& g, cudaStream_t st) {
+    const int F = head.F, K = head.K;
+    // workspace: u [B, F] | du [B, F] | dz [B, K] | part [B]
+    const size_t off_du = align_up(sizeof(float) * (size_t)B * F, 256);
+    const size_t off_dz = off_du + align_up(sizeof(float) * (size_t)B * F, 256);
+    const size_t off_part = off_dz + align_up(sizeof(float) * (size_t)B * K, 256);
+    estp_status s = ws_reserve(ctx, off_part + sizeof(float2) * (size_t)B);
+    if (s != ESTP_OK) return s;
+    char* ws = static_cast<char*>(ctx->ws);
+    float* u = reinterpret_cast<float*>(ws);
+    float* du = reinterpret_cast<float*>(ws + off_du);
+    float* dz = reinterpret_cast<float*>(ws + off_dz);
+    float2* part = reinterpret_cast<float2*>(ws + off_part);
+    const bool lower = g.W1 || g.b1 || g.pooled;  // gradients below the hidden layer
+    cudaError_t e = mlp_hidden(ctx, pooled, B, D, head, u, st);
+    if (e != cudaSuccess) return cuda_fail(e, "mlp hidden launch");
+    head_fwd_kernel<<<B, kFwdThreads, 0, st>>>(u, F, head.W2, head.b2, head.centers, K, targets, B,
+                                               lambda3, dz, part, nullptr, nullptr);
+    // second layer: dL/dW2, dL/db2, dL/du and the loss
+    int64_t total = (g.W2 ? (int64_t)K * F : 0) + (g.b2 ? K : 0) + (lower ? (int64_t)B * F : 0) + 1;
+    head_grad_kernel<<<grad_blocks(ctx, total), 256, 0, st>>>(u, B, F, head.W2, K, dz, nullptr, part,
+                                                              lambda3, loss, g.W2, g.b2,
+                                                              lower ? du : nullptr);
+    if (lower) {  // first layer, through the ReLU (u > 0): dL/dW1, dL/db1, dL/dpooled
+        total = (g.W1 ? (int64_t)F * D : 0) + (g.b1 ? F : 0) + (g.pooled ? (int64_t)B * D : 0);
+        head_grad_kernel<<<grad_blocks(ctx, total), 256, 0, st>>>(pooled, B, D, head.W1, F, du, u,
+                                                                  nullptr, 0.f, nullptr, g.W1, g.b1,
+                                                                  g.pooled);
+    }
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "mlp head loss launch");
 }
 
 }  // namespace estp
