@@ -153,15 +153,23 @@ __global__ void head_grad_kernel(const float* __restrict__ pooled, int B, int64_
     }
 }
 
-constexpr int kHidB = 8;  // prompts per warp pass of the hidden layer
+constexpr int kHidB = 16;  // prompts per warp pass of the hidden layer
+constexpr int kDhB = 4;    // prompts per block of the input gradient
 
-// u[b, f] = max(sum_x W1[f, x] h[b, x] + b1[f], 0): warp w of the grid takes hidden
-// unit f = w, and the prompts kHidB at a time.
-__global__ void __launch_bounds__(256) mlp_hidden_kernel(const float* __restrict__ pooled,
-                                                         int B, int64_t D,
-                                                         const float* __restrict__ W1,
+// Four consecutive floats of a row at column x (a 16-byte load when vec, else scalar
+// loads, zero past D).
+__device__ __forceinline__ float4 ld4(const float* __restrict__ row, int64_t x, int64_t D, bool vec) {
+    if (vec) return __ldg(reinterpret_cast<const float4*>(row + x));
+    return make_float4(x < D ? __ldg(row + x) : 0.f, x + 1 < D ? __ldg(row + x + 1) : 0.f,
+                       x + 2 < D ? __ldg(row + x + 2) : 0.f, x + 3 < D ? __ldg(row + x + 3) : 0.f);
+}
+
+// u[b, f] = max(sum_x W1[f, x] h[b, x] + b1[f], 0): one warp per hidden unit f, lanes
+// stride D four columns at a time, kHidB prompts per pass, then a fixed butterfly.
+__global__ void __launch_bounds__(128) mlp_hidden_kernel(const float* __restrict__ pooled, int B,
+                                                         int64_t D, const float* __restrict__ W1,
                                                          const float* __restrict__ b1, int F,
-                                                         float* __restrict__ u) {
+                                                         float* __restrict__ u, int vec) {
     const int lane = threadIdx.x & 31;
     const int64_t f = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (f >= F) return;
@@ -172,17 +180,140 @@ __global__ void __launch_bounds__(256) mlp_hidden_kernel(const float* __restrict
         float acc[kHidB];
 #pragma unroll
         for (int j = 0; j < kHidB; ++j) acc[j] = 0.f;
-        for (int64_t x = lane; x < D; x += 32) {
-            const float wx = w[x];
+        for (int64_t x = 4 * lane; x < D; x += 128) {
+            // every load of the pass first (rows past B repeat the last row, unused), then the FMAs
+            const float4 wv = ld4(w, x, D, vec);
+            float4 hv[kHidB];
 #pragma unroll
             for (int j = 0; j < kHidB; ++j)
-                if (j < nb) acc[j] = fmaf(wx, pooled[(int64_t)(b0 + j) * D + x], acc[j]);
+                hv[j] = ld4(pooled + (int64_t)(b0 + (j < nb ? j : nb - 1)) * D, x, D, vec);
+#pragma unroll
+            for (int j = 0; j < kHidB; ++j)
+                acc[j] = fmaf(wv.x, hv[j].x, fmaf(wv.y, hv[j].y, fmaf(wv.z, hv[j].z, fmaf(wv.w, hv[j].w, acc[j]))));
         }
 #pragma unroll
         for (int j = 0; j < kHidB; ++j) {
             const float a = warp_sum(acc[j]) + bias;
             if (lane == 0 && j < nb) u[(int64_t)(b0 + j) * F + f] = a > 0.f ? a : 0.f;
         }
+    }
+}
+
+// dL/dh[b, x] = sum_f W1[f, x] g[b, f], g = dL/du where u > 0 (the ReLU's derivative), else 0.
+// Block (128 columns, kDhB prompts): g of the block's prompts is staged in shared memory
+// (dynamic, kDhB x F floats); warp w takes f = w, w + 8, ... (four W1 rows in flight);
+// the 8 warp partials are added in warp order.
+__global__ void __launch_bounds__(256) mlp_dh_kernel(const float* __restrict__ W1, int64_t D, int F,
+                                                     const float* __restrict__ du,
+                                                     const float* __restrict__ u, int B,
+                                                     float* __restrict__ dh, int vec) {
+    extern __shared__ float g_s[];  // [kDhB][F]
+    __shared__ float4 red[8][kDhB][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t x = (int64_t)blockIdx.x * 128 + 4 * lane;
+    const int b0 = blockIdx.y * kDhB;
+    const int nb = B - b0 < kDhB ? B - b0 : kDhB;
+    for (int q = threadIdx.x; q < kDhB * F; q += blockDim.x) {
+        const int j = q / F, f = q - j * F;
+        float gv = 0.f;
+        if (j < nb) {
+            const int64_t i = (int64_t)(b0 + j) * F + f;
+            gv = u[i] > 0.f ? du[i] : 0.f;
+        }
+        g_s[q] = gv;
+    }
+    __syncthreads();
+    float4 acc[kDhB];
+#pragma unroll
+    for (int j = 0; j < kDhB; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (x < D) {
+        int f = warp;
+        for (; f + 24 < F; f += 32) {  // four rows f, f + 8, f + 16, f + 24 in flight
+            float4 wv[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) wv[r] = ld4(W1 + (int64_t)(f + 8 * r) * D, x, D, vec);
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+                for (int j = 0; j < kDhB; ++j) {
+                    const float gv = g_s[j * F + f + 8 * r];
+                    acc[j].x = fmaf(gv, wv[r].x, acc[j].x);
+                    acc[j].y = fmaf(gv, wv[r].y, acc[j].y);
+                    acc[j].z = fmaf(gv, wv[r].z, acc[j].z);
+                    acc[j].w = fmaf(gv, wv[r].w, acc[j].w);
+                }
+        }
+        for (; f < F; f += 8) {
+            const float4 wv = ld4(W1 + (int64_t)f * D, x, D, vec);
+#pragma unroll
+            for (int j = 0; j < kDhB; ++j) {
+                const float gv = g_s[j * F + f];
+                acc[j].x = fmaf(gv, wv.x, acc[j].x);
+                acc[j].y = fmaf(gv, wv.y, acc[j].y);
+                acc[j].z = fmaf(gv, wv.z, acc[j].z);
+                acc[j].w = fmaf(gv, wv.w, acc[j].w);
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kDhB; ++j) red[warp][j][lane] = acc[j];
+    __syncthreads();
+    if (warp == 0 && x < D) {
+        for (int j = 0; j < nb; ++j) {
+            float4 t = red[0][j][lane];
+            for (int w = 1; w < 8; ++w) {
+                const float4 o = red[w][j][lane];
+                t.x += o.x;
+                t.y += o.y;
+                t.z += o.z;
+                t.w += o.w;
+            }
+            float* out = dh + (int64_t)(b0 + j) * D + x;
+            out[0] = t.x;
+            if (x + 1 < D) out[1] = t.y;
+            if (x + 2 < D) out[2] = t.z;
+            if (x + 3 < D) out[3] = t.w;
+        }
+    }
+}
+
+// dL/dW1[f, x] = sum_b g[b, f] h[b, x] and dL/db1[f] = sum_b g[b, f], g = dL/du where u > 0:
+// thread (f, four columns x) sums the prompts in order; the threads with x = 0 also write
+// dL/db1[f].  Either output may be NULL.
+__global__ void __launch_bounds__(256) mlp_dw1_kernel(const float* __restrict__ pooled, int B,
+                                                      int64_t D, int F, const float* __restrict__ du,
+                                                      const float* __restrict__ u,
+                                                      float* __restrict__ gW1,
+                                                      float* __restrict__ gb1, int vec) {
+    const int64_t per_row = (D + 3) / 4;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= (int64_t)F * per_row) return;
+    const int f = (int)(t / per_row);
+    const int64_t x = 4 * (t - (int64_t)f * per_row);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float gs = 0.f;
+    for (int b = 0; b < B; ++b) {
+        const int64_t i = (int64_t)b * F + f;
+        const float gv = u[i] > 0.f ? du[i] : 0.f;
+        gs += gv;
+        if (gW1) {
+            const float4 hv = ld4(pooled + (int64_t)b * D, x, D, vec);
+            acc.x = fmaf(gv, hv.x, acc.x);
+            acc.y = fmaf(gv, hv.y, acc.y);
+            acc.z = fmaf(gv, hv.z, acc.z);
+            acc.w = fmaf(gv, hv.w, acc.w);
+        }
+    }
+    if (gb1 && x == 0) gb1[f] = gs;
+    if (!gW1) return;
+    float* out = gW1 + (int64_t)f * D + x;
+    if (vec) {
+        *reinterpret_cast<float4*>(out) = acc;
+    } else {
+        out[0] = acc.x;
+        if (x + 1 < D) out[1] = acc.y;
+        if (x + 2 < D) out[2] = acc.z;
+        if (x + 3 < D) out[3] = acc.w;
     }
 }
 
@@ -216,11 +347,15 @@ estp_status launch_head_loss(estp_ctx* ctx, const float* pooled, int B, int64_t 
 }
 
 // The MLP's hidden units u [B, F] into the workspace at `u`.
+static bool vec4(const float* a, const float* b, int64_t D) {
+    return D % 4 == 0 && aligned16(a) && aligned16(b);
+}
+
 static cudaError_t mlp_hidden(estp_ctx* ctx, const float* pooled, int B, int64_t D,
                               const estp_mlp_head& head, float* u, cudaStream_t st) {
     const int64_t threads = 32 * (int64_t)head.F;
-    mlp_hidden_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(pooled, B, D, head.W1,
-                                                                        head.b1, head.F, u);
+    mlp_hidden_kernel<<<(unsigned)((threads + 127) / 128), 128, 0, st>>>(
+        pooled, B, D, head.W1, head.b1, head.F, u, vec4(pooled, head.W1, D) ? 1 : 0);
     return cudaGetLastError();
 }
 
@@ -263,11 +398,25 @@ estp_status launch_mlp_head_loss(estp_ctx* ctx, const float* pooled, int B, int6
     head_grad_kernel<<<grad_blocks(ctx, total), 256, 0, st>>>(u, B, F, head.W2, K, dz, nullptr, part,
                                                               lambda3, loss, g.W2, g.b2,
                                                               lower ? du : nullptr);
-    if (lower) {  // first layer, through the ReLU (u > 0): dL/dW1, dL/db1, dL/dpooled
-        total = (g.W1 ? (int64_t)F * D : 0) + (g.b1 ? F : 0) + (g.pooled ? (int64_t)B * D : 0);
+    if (g.W1 || g.b1) {  // first layer, through the ReLU (u > 0): dL/dW1, dL/db1
+        const int64_t threads = (int64_t)F * ((D + 3) / 4);
+        mlp_dw1_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(
+            pooled, B, D, F, du, u, g.W1, g.b1, vec4(pooled, g.W1 ? g.W1 : pooled, D) ? 1 : 0);
+    }
+    const size_t smem = sizeof(float) * kDhB * (size_t)F;
+    if (g.pooled && smem > 200 * 1024) {  // very wide hidden layer: the general kernel
+        total = (int64_t)B * D;
         head_grad_kernel<<<grad_blocks(ctx, total), 256, 0, st>>>(pooled, B, D, head.W1, F, du, u,
-                                                                  nullptr, 0.f, nullptr, g.W1, g.b1,
-                                                                  g.pooled);
+                                                                  nullptr, 0.f, nullptr, nullptr,
+                                                                  nullptr, g.pooled);
+    } else if (g.pooled) {  // dL/dpooled = W1^T (dL/du where u > 0)
+        const dim3 grid((unsigned)((D + 127) / 128), (unsigned)((B + kDhB - 1) / kDhB));
+        if (smem > 48 * 1024) {
+            e = cudaFuncSetAttribute(mlp_dh_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return cuda_fail(e, "mlp input-gradient smem attribute");
+        }
+        mlp_dh_kernel<<<grid, 256, smem, st>>>(head.W1, D, F, du, u, B, g.pooled,
+                                               vec4(head.W1, head.W1, D) ? 1 : 0);
     }
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "mlp head loss launch");

@@ -48,7 +48,8 @@ def _dev(cuda_lib, W1, b1, W2, b2, c):
 
 @pytest.mark.parametrize("lam", [0.0, 0.5, 1.0])
 @pytest.mark.parametrize("B,D,F,K", [(16, 3584, 1024, 32), (1, 512, 64, 32), (5, 64, 7, 1),
-                                     (3, 33, 300, 1000), (9, 100, 1, 5)])
+                                     (3, 33, 300, 1000), (9, 100, 1, 5), (19, 130, 37, 3),
+                                     (2, 64, 13000, 4)])
 def test_mlp_loss_against_oracle(cuda_lib, B, D, F, K, lam):
     h, W1, b1, W2, b2, c, y = _case(B, D, F, K)
     ctx = cuda_lib.Context(0)
