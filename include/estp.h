@@ -47,7 +47,7 @@ typedef struct CUstream_st* estp_stream_t; /* same type as cudaStream_t */
 typedef enum {
     ESTP_OK = 0,
     ESTP_ERR_INVALID_ARG = 1,  /* bad size, pointer, alignment or varlen metadata */
-    ESTP_ERR_UNSUPPORTED = 2,  /* valid request this build does not implement     */
+    ESTP_ERR_UNSUPPORTED = 2,  /* valid request the library does not implement   */
     ESTP_ERR_CUDA = 3,         /* a CUDA runtime call failed (message in last_error) */
     ESTP_ERR_TIMEOUT = 4,      /* a device-side bounded wait gave up               */
     ESTP_ERR_WORKSPACE = 5     /* workspace could not be (re)allocated             */
