@@ -23,11 +23,7 @@
 //
 // Every mbarrier wait is bounded; on expiry the CTA records ESTP_ERR_TIMEOUT in the status
 // word, drains its own copies and MMAs and frees its TMEM.
-#include <cuda.h>
-#include <cudaTypedefs.h>
-
-#include "estp_internal.cuh"
-#include "ptx.cuh"
+#include "tcgen05.cuh"
 
 namespace estp {
 namespace {
@@ -50,10 +46,8 @@ constexpr int kMiscOff = kBarOff + kNumBars * 8;           // tmem address, abor
 constexpr int kSmemBytes = kMiscOff + 16 + 1024;           // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
-// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both K-major,
-// N = 256, M = 128.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kN >> 3) << 17) |
-                            ((uint32_t)(kM >> 4) << 24);
+// Instruction descriptor: M = 128, N = 256.
+constexpr uint32_t kIdesc = idesc_bf16(kM, kN);
 
 struct LmArgs {
     int64_t n_rows;
@@ -65,66 +59,6 @@ struct LmArgs {
     float* part;       // [3][S][n_rows]: m, s, t (log2 units)
     int* status;
 };
-
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
-                                            uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups
-// 1024 bytes apart, descriptor version 1.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
-    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
-           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(kIdesc), "r"(acc));
-}
-
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-            smem_u32(bar))
-        : "memory");
-}
-
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-        "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
-        "%28, %29, %30, %31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31])
-        : "r"(taddr));
-#pragma unroll
-    for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
-}
-
-__device__ __forceinline__ void tmem_wait_ld() {
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 // Vocabulary tiles [vt0, vt1) of split sp.
 __device__ __forceinline__ void split_range(const LmArgs& a, int sp, int& vt0, int& vt1) {
@@ -273,7 +207,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t sa = smem_u32(sm + stage * kStageBytes);
 #pragma unroll
                         for (int kk = 0; kk < kKc / 16; ++kk)
-                            mma_bf16(d, sw128_desc(sa + kk * 32), sw128_desc(sa + kABytes + kk * 32),
+                            mma_bf16<kIdesc>(d, sw128_desc(sa + kk * 32), sw128_desc(sa + kABytes + kk * 32),
                                      (kc > 0 || kk > 0) ? 1u : 0u);
                         mma_commit(&empty[stage]);
                     }
@@ -362,24 +296,12 @@ __global__ void lm_head_merge_kernel(const float* __restrict__ part, int64_t n_r
     H[r] = kLn2 * (lg2(Sx) - Tx / Sx);
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }
-    return fn;
-}
 
 // [rows, ld] bf16 row-major viewed as a 2-D tensor (D, rows); box 64 x box_rows, 128B
 // swizzle; rows past the end read as zero.
 estp_status make_map_2d(CUtensorMap* m, const void* base, int64_t D, int64_t rows, int64_t ld,
                         int box_rows) {
-    auto fn = encode_fn();
+    auto fn = tensor_map_encoder();
     if (!fn) return fail(ESTP_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
     cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
