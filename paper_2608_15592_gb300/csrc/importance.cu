@@ -289,9 +289,18 @@ __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const
         const int T = cuv[b + 1] - cuv[b];
         const int nt = (T + tile - 1) / tile;
         const int kt = (int)((j - cuv[b]) / tile);
-        const int nch = chunks_of(nt, kt, qc);
-        for (int c = 0; c < nch; ++c)
-            for (int g = 0; g < n_groups; ++g) v += part[((int64_t)c * n_groups + g) * sumT + j];
+        const int n = chunks_of(nt, kt, qc) * n_groups;  // partials (c, g), c-major
+        // up to 16 partials are loaded before any is added (independent loads in flight),
+        // then added in the same (c, g) order
+        constexpr int kBatch = 16;
+        for (int i0 = 0; i0 < n; i0 += kBatch) {
+            float p[kBatch];
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) p[i] = i0 + i < n ? part[(int64_t)(i0 + i) * sumT + j] : 0.f;
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i)
+                if (i0 + i < n) v += p[i];
+        }
     }
     acc[j] = accumulate ? acc[j] + v : v;
 }
