@@ -19,20 +19,9 @@
 namespace estp {
 namespace {
 
-#ifndef ESTP_ENT_UNROLL
-#define ESTP_ENT_UNROLL 8
-#endif
-#ifndef ESTP_ENT_MINB
-#define ESTP_ENT_MINB 3
-#endif
-#ifndef ESTP_ENT_PACKED   // 1: packed f32x2 FMA/ADD; 0: scalar FMA/ADD
-#define ESTP_ENT_PACKED 0
-#endif
-#ifndef ESTP_ENT_PREFETCH // 1: next batch loaded while the current one is reduced
-#define ESTP_ENT_PREFETCH 0
-#endif
 constexpr int kEntThreads = 256;
-constexpr int kEntUnroll = ESTP_ENT_UNROLL;  // 16-byte loads per lane per batch (two batches in flight)
+constexpr int kEntMinBlocks = 3;  // resident blocks per SM the registers are sized for
+constexpr int kEntUnroll = 8;     // 16-byte loads per lane per batch
 constexpr float kMaskedLogit = -1e30f;  // finite: 2^(masked - m) = 0 and 0 * d = 0
 
 struct EntPart {
@@ -60,25 +49,6 @@ __device__ __forceinline__ int64_t unit_owner(int64_t units, int64_t W, int64_t 
     return w < W - 1 ? w : W - 1;
 }
 
-// Online update with the batch max already folded into m.
-__device__ __forceinline__ void rescale(float& m, float2& s, float2& t, float new_m) {
-    float dm = m - new_m;  // <= 0
-    float f = ex2(dm);
-    t.x = f * fmaf(dm, s.x, t.x);
-    t.y = f * fmaf(dm, s.y, t.y);
-    s.x *= f;
-    s.y *= f;
-    m = new_m;
-}
-
-__device__ __forceinline__ void accum_pair(float2 x, float m, float2& s, float2& t) {
-    const float2 l2e = make_float2(kLog2e, kLog2e);
-    const float2 nm = make_float2(-m, -m);
-    float2 d = __ffma2_rn(x, l2e, nm);  // y - m
-    float2 e = make_float2(ex2(d.x), ex2(d.y));
-    s = __fadd2_rn(s, e);
-    t = __ffma2_rn(e, d, t);
-}
 
 __device__ __forceinline__ void merge(float& m, float& s, float& t, float m2, float s2, float t2) {
     float mm = fmaxf(m, m2);
@@ -183,17 +153,7 @@ __device__ __forceinline__ void reduce_batch(const uint4* v, float& m, float2& s
     m = new_m;
 #pragma unroll
     for (int k = 0; k < kEntUnroll; ++k) {
-        if (ESTP_ENT_PACKED) {
-            if (kBf16) {
-                accum_pair(make_float2(bf16lo(v[k].x), bf16hi(v[k].x)), m, s, t);
-                accum_pair(make_float2(bf16lo(v[k].y), bf16hi(v[k].y)), m, s1, t1);
-                accum_pair(make_float2(bf16lo(v[k].z), bf16hi(v[k].z)), m, s, t);
-                accum_pair(make_float2(bf16lo(v[k].w), bf16hi(v[k].w)), m, s1, t1);
-            } else {
-                accum_pair(make_float2(__uint_as_float(v[k].x), __uint_as_float(v[k].y)), m, s, t);
-                accum_pair(make_float2(__uint_as_float(v[k].z), __uint_as_float(v[k].w)), m, s1, t1);
-            }
-        } else if (kBf16) {  // four independent (s, t) chains
+        if (kBf16) {  // four independent (s, t) chains
             accum1(bf16lo(v[k].x), m, s.x, t.x);
             accum1(bf16hi(v[k].x), m, s.y, t.y);
             accum1(bf16lo(v[k].y), m, s1.x, t1.x);
@@ -211,8 +171,6 @@ __device__ __forceinline__ void reduce_batch(const uint4* v, float& m, float2& s
     }
 }
 
-// One lane's share of units [c0, c1) of one row (lane handles c0 + lane + 32k), with
-// the next batch's loads issued before the current batch is reduced.
 // One lane's share of units [c0, c1) of one row (lane handles c0 + lane + 32k).
 // Full batches run without bounds checks through a moving pointer; the ragged
 // remainder and the row's partial last unit (when V is not a multiple of the
@@ -228,30 +186,11 @@ __device__ __forceinline__ void segment(const char* row, int64_t c0, int64_t c1,
     const int64_t c1m = (c1 == nvec && tail_valid < kPerUnit) ? c1 - 1 : c1;
     int64_t c = c0 + lane;
     const uint4* p = reinterpret_cast<const uint4*>(row) + c;
-    if (ESTP_ENT_PREFETCH && c + kStride * 2 - 32 < c1m) {
-        uint4 va[kEntUnroll], vb[kEntUnroll];
+    for (; c + kStride - 32 < c1m; c += kStride, p += kStride) {
+        uint4 v[kEntUnroll];
 #pragma unroll
-        for (int k = 0; k < kEntUnroll; ++k) va[k] = ld_stream(p + 32 * k);
-        while (true) {
-            p += kStride;
-            c += kStride;
-            const bool more = c + kStride - 32 < c1m;
-            if (more) {
-#pragma unroll
-                for (int k = 0; k < kEntUnroll; ++k) vb[k] = ld_stream(p + 32 * k);
-            }
-            reduce_batch<kBf16>(va, m, s, t, s1, t1);
-            if (!more) break;
-#pragma unroll
-            for (int k = 0; k < kEntUnroll; ++k) va[k] = vb[k];
-        }
-    } else {
-        for (; c + kStride - 32 < c1m; c += kStride, p += kStride) {
-            uint4 v[kEntUnroll];
-#pragma unroll
-            for (int k = 0; k < kEntUnroll; ++k) v[k] = ld_stream(p + 32 * k);
-            reduce_batch<kBf16>(v, m, s, t, s1, t1);
-        }
+        for (int k = 0; k < kEntUnroll; ++k) v[k] = ld_stream(p + 32 * k);
+        reduce_batch<kBf16>(v, m, s, t, s1, t1);
     }
     if (c < c1) {  // remainder: fewer than kEntUnroll units left for this lane
         uint4 v[kEntUnroll];
@@ -263,7 +202,7 @@ __device__ __forceinline__ void segment(const char* row, int64_t c0, int64_t c1,
 }
 
 template <bool kBf16>
-__global__ void __launch_bounds__(kEntThreads, ESTP_ENT_MINB) entropy_kernel(EntArgs a) {
+__global__ void __launch_bounds__(kEntThreads, kEntMinBlocks) entropy_kernel(EntArgs a) {
     const int lane = threadIdx.x & 31;
     const int64_t w = (int64_t)blockIdx.x * (kEntThreads / 32) + (threadIdx.x >> 5);
     if (w >= a.n_warps) return;
