@@ -9,6 +9,7 @@ Functions and the paper passages they follow (arXiv 2608.15592):
   lm_head_entropy Eq. 2-1 of the logits h W^T formed from hidden states
   attn_lse        the row normaliser of the causal softmax A (Sec. 3.1)
   attn_colsum     sum_i A_ij of Eq. 2-0 for one layer, summed over query heads
+  attn_output     O = A V, the prefill's attention output (Sec. 3.1)
   attn_colsum_rows  the same from the rows i >= row_from only (exact for late keys)
   importance      Eq. 2-0: S_j = C_j / (N * layers * heads); divisor variants of its 1/N
   pool            Eqs. 2-2, 2-3, 2-4
@@ -58,6 +59,7 @@ class _Lib:
             "oracle_token_entropy": [P, I, I64, I64, I64, P, I],
             "oracle_lm_head_entropy": [P, P, I, I64, I64, I64, I64, I64, P, I],
             "oracle_attn_lse": [P, P, I, I, I, I, D, P, I, P, I],
+            "oracle_attn_output": [P, P, P, I, I, I, I, D, P, I, P, I],
             "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
             "oracle_attn_colsum_rows": [P, P, I, I, I, I, D, P, I, P, I, I, I64, P, I],
             "oracle_importance": [P, P, I, I, I, P],
@@ -167,6 +169,20 @@ def lm_head_entropy(hidden: np.ndarray, W: np.ndarray, n_threads: int = 0) -> np
     out = np.zeros(rows, dtype=np.float64)
     _check(_load().oracle_lm_head_entropy(_ptr(hidden), _ptr(W), _dtype_code(hidden), rows, D,
                                           V, D, D, _ptr(out), n_threads), "lm_head_entropy")
+    return out
+
+
+def attn_output(Q, K, V, cu_seqlens, scale, n_threads: int = 0) -> np.ndarray:
+    """O [sumT, Hq, d] = A V of the causal attention of one layer (V read with K's head)."""
+    Q, K, V = np.ascontiguousarray(Q), np.ascontiguousarray(K), np.ascontiguousarray(V)
+    cu = _cu(cu_seqlens)
+    sumT, Hq, d = Q.shape
+    Hkv = K.shape[1]
+    assert K.shape == V.shape and K.dtype == Q.dtype == V.dtype
+    out = np.zeros((sumT, Hq, d), dtype=np.float64)
+    _check(_load().oracle_attn_output(_ptr(Q), _ptr(K), _ptr(V), _dtype_code(Q), Hq, Hkv, d,
+                                      float(scale), _ptr(cu), len(cu) - 1, _ptr(out), n_threads),
+           "attn_output")
     return out
 
 

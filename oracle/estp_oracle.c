@@ -243,6 +243,72 @@ static int64_t max_len(const int32_t* cu, int B) {
     return mx;
 }
 
+/* ------------------------------- the attention output of the prefill (Sec. 3.1) */
+
+typedef struct {
+    const void *Q, *K, *V;
+    int dtype, Hq, Hkv, d;
+    double scale;
+    const int32_t* cu;
+    double* O;
+} attn_out_ctx;
+
+/* One (prompt, query head) pair: for every query row i, the causal softmax row
+ * A_ij = exp(s_ij - m) / Z over the keys j <= i, s_ij = scale * q_i . k_j, and the
+ * attention output O_i = sum_j A_ij v_j (V read with K's head). scratch: >= T doubles. */
+static void attn_out_unit(void* vctx, int64_t unit, double* s) {
+    attn_out_ctx* c = (attn_out_ctx*)vctx;
+    const int b = (int)(unit / c->Hq), h = (int)(unit % c->Hq), g = h / (c->Hq / c->Hkv);
+    const int64_t t0 = c->cu[b], T = (int64_t)c->cu[b + 1] - c->cu[b];
+    const int d = c->d;
+    if (T == 0) return;
+    double* q = (double*)malloc(sizeof(double) * (size_t)(T * d));
+    double* k = (double*)malloc(sizeof(double) * (size_t)(T * d));
+    double* v = (double*)malloc(sizeof(double) * (size_t)(T * d));
+    for (int64_t t = 0; t < T; ++t) {
+        const int64_t row_q = (t0 + t) * (int64_t)c->Hq + h;    /* token t, query head h */
+        const int64_t row_kv = (t0 + t) * (int64_t)c->Hkv + g;  /* token t, its KV head */
+        for (int x = 0; x < d; ++x) {
+            q[t * d + x] = load_elem(c->Q, c->dtype, row_q * d + x);
+            k[t * d + x] = load_elem(c->K, c->dtype, row_kv * d + x);
+            v[t * d + x] = load_elem(c->V, c->dtype, row_kv * d + x);
+        }
+    }
+    for (int64_t i = 0; i < T; ++i) {
+        double m = -INFINITY;
+        for (int64_t j = 0; j <= i; ++j) {
+            double dot = 0.0;
+            for (int x = 0; x < d; ++x) dot += q[i * d + x] * k[j * d + x];
+            s[j] = dot * c->scale;
+            if (s[j] > m) m = s[j];
+        }
+        double Z = 0.0;
+        for (int64_t j = 0; j <= i; ++j) Z += exp(s[j] - m);
+        double* o = c->O + ((t0 + i) * c->Hq + h) * (int64_t)d;
+        for (int x = 0; x < d; ++x) o[x] = 0.0;
+        for (int64_t j = 0; j <= i; ++j) {
+            const double a = exp(s[j] - m) / Z;
+            for (int x = 0; x < d; ++x) o[x] += a * v[j * d + x];
+        }
+    }
+    free(q);
+    free(k);
+    free(v);
+}
+
+int oracle_attn_output(const void* Q, const void* K, const void* V, int dtype, int Hq, int Hkv,
+                       int d, double scale, const int32_t* cu_seqlens, int B, double* O_out,
+                       int n_threads) {
+    if (!valid_dtype(dtype) || Hq <= 0 || Hkv <= 0 || Hq % Hkv || d <= 0) return -1;
+    if (!valid_cu(cu_seqlens, B)) return -1;
+    const int64_t sumT = cu_seqlens[B];
+    if (sumT == 0) return 0;
+    if (!Q || !K || !V || !O_out) return -1;
+    attn_out_ctx c = {Q, K, V, dtype, Hq, Hkv, d, scale, cu_seqlens, O_out};
+    parallel_units(attn_out_unit, &c, (int64_t)B * Hq, (size_t)max_len(cu_seqlens, B), n_threads);
+    return 0;
+}
+
 int oracle_attn_lse(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
                     double scale, const int32_t* cu_seqlens, int B, double* lse_out,
                     int n_threads) {

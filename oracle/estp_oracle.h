@@ -13,6 +13,7 @@
  *   oracle_lm_head_entropy     Eq. 2-1 of the logits h W^T of the output projection
  *   oracle_attn_lse            log-normaliser of the softmax rows of A (Sec. 3.1)
  *   oracle_attn_colsum         the column sums of A inside Eq. 2-0 (Sec. 3.1)
+ *   oracle_attn_output         the attention output O = A V of the prefill (Sec. 3.1)
  *   oracle_importance          Eq. 2-0 (the 1/N scaling and the head/layer mean)
  *   oracle_importance_div      Eq. 2-0 with the causal-count or no divisor (variants)
  *   oracle_pool                Eqs. 2-2, 2-3, 2-4 (Sec. 3.2)
@@ -60,6 +61,13 @@ int oracle_lm_head_entropy(const void* hidden, const void* W, int dtype, int64_t
 int oracle_attn_lse(const void* Q, const void* K, int dtype, int Hq, int Hkv, int d,
                     double scale, const int32_t* cu_seqlens, int B, double* lse_out,
                     int n_threads);
+
+/* The output of causal attention for one layer (the prefill's own attention, whose softmax
+ * rows A are those of Eq. 2-0): O[i, h, :] = sum_{j <= i, j in prompt(i)} A^h_ij V[j, h/rep, :].
+ * Q: [sumT, Hq, d], K, V: [sumT, Hkv, d] row-major; O_out: [sumT, Hq, d]. */
+int oracle_attn_output(const void* Q, const void* K, const void* V, int dtype, int Hq, int Hkv,
+                       int d, double scale, const int32_t* cu_seqlens, int B, double* O_out,
+                       int n_threads);
 
 /* Column sums of the causal softmax attention matrix of one layer, over a set of
  * query heads:  C_out[j] += sum_{h in heads} sum_{i >= j, i in prompt(j)} A^h_ij,

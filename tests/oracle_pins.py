@@ -183,6 +183,57 @@ def _qk(rng, cu, Hq, Hkv, d, spread=1.0, dtype=np.float32):
     return Q, K
 
 
+def pin_attn_output_rows_and_uniform():
+    """Attention output O = A V (Sec. 3.1): softmax rows sum to 1, so V = 1 gives O = 1;
+    Q = 0 makes every causal row uniform, so O_i is the running mean of v_0 .. v_i (numpy
+    cumulative sums), per prompt and per KV head of each query head."""
+    rng = _rng(61)
+    cu = np.array([0, 5, 5, 21, 22], np.int32)
+    Hq, Hkv, d = 6, 2, 8
+    sumT = int(cu[-1])
+    Q = rng.standard_normal((sumT, Hq, d)).astype(np.float32)
+    K = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+    ones = np.ones((sumT, Hkv, d), np.float32)
+    _close(oracle.attn_output(Q, K, ones, cu, 0.4), np.ones((sumT, Hq, d)), rtol=1e-12,
+           what="V = 1")
+    V = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+    O = oracle.attn_output(np.zeros_like(Q), K, V, cu, 0.4)
+    ref = np.zeros((sumT, Hq, d))
+    for b in range(len(cu) - 1):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        if t1 == t0:
+            continue
+        cum = np.cumsum(V[t0:t1].astype(np.float64), axis=0) / np.arange(1, t1 - t0 + 1)[:, None, None]
+        for h in range(Hq):
+            ref[t0:t1, h] = cum[:, h // (Hq // Hkv)]
+    _close(O, ref, rtol=1e-12, atol=1e-12, what="uniform rows: running mean")
+
+
+def pin_attn_output_bruteforce():
+    """T <= 16: the full masked score matrix, scipy softmax rows, times V (numpy)."""
+    rng = _rng(62)
+    for cu, Hq, Hkv, d in (([0, 16], 2, 2, 8), ([0, 3, 3, 12, 13], 4, 2, 16)):
+        cu = np.asarray(cu, np.int32)
+        sumT = int(cu[-1])
+        Q = rng.standard_normal((sumT, Hq, d)).astype(np.float32)
+        K = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+        V = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+        scale = 1 / math.sqrt(d)
+        ref = np.zeros((sumT, Hq, d))
+        for b in range(len(cu) - 1):
+            t0, t1 = int(cu[b]), int(cu[b + 1])
+            T = t1 - t0
+            if T == 0:
+                continue
+            for h in range(Hq):
+                g = h // (Hq // Hkv)
+                s = scale * Q[t0:t1, h].astype(np.float64) @ K[t0:t1, g].astype(np.float64).T
+                s[np.triu_indices(T, 1)] = -np.inf
+                ref[t0:t1, h] = special.softmax(s, axis=1) @ V[t0:t1, g].astype(np.float64)
+        _close(oracle.attn_output(Q, K, V, cu, scale), ref, rtol=1e-12, atol=1e-12,
+               what="attention output brute force")
+
+
 def pin_importance_bruteforce():
     """T <= 16: column sums of scipy softmax rows of the causal score matrix."""
     rng = _rng(3)

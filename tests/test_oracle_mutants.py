@@ -29,6 +29,15 @@ MUTANTS = [
     ("Q prompt offset dropped", "((t0 + t) * c->Hq + h)", "((t) * c->Hq + h)"),
     ("self term never excluded", "if (c->exclude_self && j == i) continue;", ""),
     ("lse sign", "m + log(Z);", "m - log(Z);"),
+    ("output scores unscaled", "s[j] = dot * c->scale;", "s[j] = dot;"),
+    ("output weights unnormalised", "const double a = exp(s[j] - m) / Z;",
+     "const double a = exp(s[j] - m);"),
+    ("output reads the key rows as values", "v[t * d + x] = load_elem(c->V,",
+     "v[t * d + x] = load_elem(c->K,"),
+    ("output ignores the GQA map", "const int64_t row_kv = (t0 + t) * (int64_t)c->Hkv + g;",
+     "const int64_t row_kv = (t0 + t) * (int64_t)c->Hkv + 0;"),
+    ("output drops the diagonal", "for (int64_t j = 0; j <= i; ++j) {\n            const double a",
+     "for (int64_t j = 0; j < i; ++j) {\n            const double a"),
     ("rows_from off by one", "for (int64_t i = c->row_from; i < T; ++i) {",
      "for (int64_t i = c->row_from + 1; i < T; ++i) {"),
     ("causal count divisor", "if (divisor == ORACLE_DIV_LENGTH) n = (double)N;",
