@@ -178,6 +178,31 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
                                  int64_t sumT, int32_t max_seqlen, int accumulate,
                                  uint32_t flags, estp_stream_t stream);
 
+/* The prefill's causal attention output with the importance column sums of the same
+ * probabilities (Sec. 3.1: the attention maps of the prefill; Eq. 2-0), one layer per call:
+ *   out[i, h, :] = sum_{j <= i, j in prompt(i)} A^h_ij V[j, h / (Hq / Hkv), :]
+ *   C_j (+)= sum_{h < Hq} sum_{i >= j, i in prompt(j)} A^h_ij
+ * with A^h_ij = exp(s_ij - lse_i) as in estp_attn_lse.  The importance side is that of
+ * estp_attn_importance over all Hq heads (same accumulation, same flags, closed by
+ * estp_attn_importance_finalize); the two entry points may be mixed within one
+ * accumulation as long as every call covers all Hq heads.
+ *   Q   : bf16 [sumT, Hq, 128];  K, V : bf16 [sumT, Hkv, 128] (device, 16-byte aligned)
+ *   lse : fp32 [Hq, sumT] (the prefill's, or estp_attn_lse's), or NULL to have the library
+ *         compute it first.
+ *   out : bf16 [sumT, Hq, 128] (device, 16-byte aligned), written for every token.
+ *   dtype must be ESTP_BF16 and head_dim 128 (else ESTP_ERR_UNSUPPORTED).
+ * The probabilities enter O = A V rounded to bf16 (as a flash-attention forward does);
+ * the column sums use them unrounded.  The workspace holds V^T (2 * Hkv * 128 bytes per
+ * position, prompts padded to 128) and one fp32 row of 128 column sums per (head, query
+ * tile, key tile <= query tile). */
+estp_status estp_attn_forward_importance(estp_ctx* ctx, const void* Q, const void* K,
+                                         const void* V, estp_dtype dtype, const float* lse,
+                                         int32_t Hq, int32_t Hkv, int32_t head_dim,
+                                         float softmax_scale, const int32_t* cu_seqlens,
+                                         int32_t B, int64_t sumT, int32_t max_seqlen,
+                                         int accumulate, uint32_t flags, void* out,
+                                         estp_stream_t stream);
+
 /* Ends an accumulation: importance_out[j] = C_j / (N_b * n_layers * n_heads), N_b
  * the length of the prompt holding token j (Eq. 2-0's 1/N, then the mean over the
  * selected layers and heads); N_b is replaced by the causal count n_j, or by 1, when

@@ -37,7 +37,7 @@ EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
            "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
            "estp_head_loss", "estp_misalignment", "estp_lm_head_entropy",
-           "estp_mlp_head_predict", "estp_mlp_head_loss")
+           "estp_mlp_head_predict", "estp_mlp_head_loss", "estp_attn_forward_importance")
 
 
 class EstpError(RuntimeError):
@@ -86,6 +86,8 @@ def _load():
         "estp_attn_importance": ([P, P, P, ctypes.c_int, P, I32, I32, I32, F, P, I32, P, I32,
                                   I64, I32, ctypes.c_int, U32, P], ctypes.c_int),
         "estp_attn_importance_finalize": ([P, I32, P, P], ctypes.c_int),
+        "estp_attn_forward_importance": ([P, P, P, P, ctypes.c_int, P, I32, I32, I32, F, P, I32,
+                                          I64, I32, ctypes.c_int, U32, P, P], ctypes.c_int),
         "estp_token_entropy_noalloc": ([P, ctypes.c_int, I64, I64, I64, P, P], ctypes.c_int),
         "estp_pool": ([P, P, ctypes.c_int, I64, I64, P, P, P, I32, I64, MixParams,
                        ctypes.POINTER(_Head), P, P, P], ctypes.c_int),
@@ -242,6 +244,26 @@ class Context:
                                         (ESTP_IMP_EXCLUDE_SELF if exclude_self else 0)
                                         | _DIVISOR_FLAGS[divisor],
                                         _stream(stream)))
+
+    def attn_forward_importance(self, Q, K, V, cu_seqlens, max_seqlen: int, lse=None,
+                                scale: float | None = None, accumulate: bool = False,
+                                exclude_self: bool = False, divisor: str = "length", out=None,
+                                stream=None):
+        """estp_attn_forward_importance for one layer: returns the attention output bf16
+        [sumT, Hq, 128] and adds the column sums of all Hq heads into the context's
+        importance accumulation (same accumulation and flags as attn_importance)."""
+        import torch
+        sumT, Hq, d = Q.shape
+        Hkv = K.shape[1]
+        scale = 1.0 / math.sqrt(d) if scale is None else scale
+        if out is None:
+            out = torch.empty(sumT, Hq, d, dtype=Q.dtype, device=Q.device)
+        _check(lib.estp_attn_forward_importance(
+            self._h, _ptr(Q), _ptr(K), _ptr(V), _dtype(Q), _ptr(lse), Hq, Hkv, d, scale,
+            _ptr(cu_seqlens), cu_seqlens.numel() - 1, sumT, max_seqlen, 1 if accumulate else 0,
+            (ESTP_IMP_EXCLUDE_SELF if exclude_self else 0) | _DIVISOR_FLAGS[divisor], _ptr(out),
+            _stream(stream)))
+        return out
 
     def attn_importance_finalize(self, n_layers: int, sumT: int, device=None, out=None,
                                  stream=None):

@@ -210,27 +210,22 @@ estp_status estp_attn_lse(estp_ctx* ctx, const void* Q, const void* K, estp_dtyp
                       sumT, max_seqlen, lse_out, reinterpret_cast<cudaStream_t>(stream));
 }
 
-estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
-                                 estp_dtype dtype, const float* lse, int32_t Hq, int32_t Hkv,
-                                 int32_t head_dim, float softmax_scale, const int32_t* heads,
-                                 int32_t n_heads, const int32_t* cu_seqlens, int32_t B,
-                                 int64_t sumT, int32_t max_seqlen, int accumulate,
-                                 uint32_t flags, estp_stream_t stream) {
-    estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
-                                B, sumT, max_seqlen);
-    if (st != ESTP_OK) return st;
+// Opens (accumulate = 0) or continues (accumulate = 1) the context's importance
+// accumulation over n_heads heads; checks the flags and the lse alignment, sets the device
+// and sizes the accumulator.
+static estp_status open_importance(estp_ctx* ctx, const float* lse, int n_heads,
+                                   const int32_t* cu_seqlens, int32_t B, int64_t sumT,
+                                   int accumulate, uint32_t flags) {
     constexpr uint32_t kDiv = ESTP_IMP_DIV_CAUSAL | ESTP_IMP_DIV_NONE;
     if (flags & ~(ESTP_IMP_EXCLUDE_SELF | kDiv)) return fail(ESTP_ERR_INVALID_ARG, "unknown flags");
     if ((flags & kDiv) == kDiv)
         return fail(ESTP_ERR_INVALID_ARG, "ESTP_IMP_DIV_CAUSAL and ESTP_IMP_DIV_NONE together");
-    ImpHeads hs;
-    st = build_heads(heads, n_heads, Hq, Hkv, &hs);
-    if (st != ESTP_OK) return st;
+    estp_status st;
     if (accumulate) {
         if (!ctx->imp_open)
             return fail(ESTP_ERR_INVALID_ARG, "accumulate=1 without an open accumulation");
         if (ctx->imp_sumT != sumT || ctx->imp_B != B || ctx->imp_cu != cu_seqlens ||
-            ctx->imp_n_heads != hs.n_heads)
+            ctx->imp_n_heads != n_heads)
             return fail(ESTP_ERR_INVALID_ARG,
                         "accumulate=1 with different cu_seqlens/B/sumT/head count");
         // the finalize divisor is fixed when the accumulation opens; the causal count
@@ -260,12 +255,52 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
     ctx->imp_sumT = sumT;
     ctx->imp_B = B;
     ctx->imp_cu = cu_seqlens;
-    ctx->imp_n_heads = hs.n_heads;
+    ctx->imp_n_heads = n_heads;
     if (!accumulate) ctx->imp_flags = flags;
+    return ESTP_OK;
+}
+
+estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
+                                 estp_dtype dtype, const float* lse, int32_t Hq, int32_t Hkv,
+                                 int32_t head_dim, float softmax_scale, const int32_t* heads,
+                                 int32_t n_heads, const int32_t* cu_seqlens, int32_t B,
+                                 int64_t sumT, int32_t max_seqlen, int accumulate,
+                                 uint32_t flags, estp_stream_t stream) {
+    estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
+                                B, sumT, max_seqlen);
+    if (st != ESTP_OK) return st;
+    ImpHeads hs;
+    st = build_heads(heads, n_heads, Hq, Hkv, &hs);
+    if (st != ESTP_OK) return st;
+    st = open_importance(ctx, lse, hs.n_heads, cu_seqlens, B, sumT, accumulate, flags);
+    if (st != ESTP_OK) return st;
     if (sumT == 0 || B == 0) return ESTP_OK;
     return launch_importance(ctx, Q, K, dtype, lse, Hq, Hkv, head_dim, softmax_scale, hs,
                              cu_seqlens, B, sumT, max_seqlen, accumulate != 0, flags,
                              ctx->imp_acc, reinterpret_cast<cudaStream_t>(stream));
+}
+
+estp_status estp_attn_forward_importance(estp_ctx* ctx, const void* Q, const void* K,
+                                         const void* V, estp_dtype dtype, const float* lse,
+                                         int32_t Hq, int32_t Hkv, int32_t head_dim,
+                                         float softmax_scale, const int32_t* cu_seqlens,
+                                         int32_t B, int64_t sumT, int32_t max_seqlen,
+                                         int accumulate, uint32_t flags, void* out,
+                                         estp_stream_t stream) {
+    estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
+                                B, sumT, max_seqlen);
+    if (st != ESTP_OK) return st;
+    if (dtype != ESTP_BF16) return fail(ESTP_ERR_UNSUPPORTED, "attention forward: bf16 only");
+    if (head_dim != 128) return fail(ESTP_ERR_UNSUPPORTED, "attention forward: head_dim 128 only");
+    if (sumT > 0 && (!V || !out)) return fail(ESTP_ERR_INVALID_ARG, "NULL V or out");
+    if (sumT > 0 && (!aligned16(V) || !aligned16(out)))
+        return fail(ESTP_ERR_INVALID_ARG, "V and out must be 16-byte aligned");
+    st = open_importance(ctx, lse, Hq, cu_seqlens, B, sumT, accumulate, flags);
+    if (st != ESTP_OK) return st;
+    if (sumT == 0 || B == 0) return ESTP_OK;
+    return launch_attn_forward(ctx, Q, K, V, lse, Hq, Hkv, softmax_scale, cu_seqlens, B, sumT,
+                               max_seqlen, (flags & ESTP_IMP_EXCLUDE_SELF) != 0, accumulate != 0,
+                               ctx->imp_acc, out, reinterpret_cast<cudaStream_t>(stream));
 }
 
 estp_status estp_attn_importance_finalize(estp_ctx* ctx, int32_t n_layers,

@@ -1,0 +1,596 @@
+// The prefill's causal attention output with the importance column sums taken from the
+// same probability tiles (Sec. 3.1, Eq. 2-0): O = A V for every query head, and
+// C_j += sum_h sum_{i >= j} A^h_ij for the importance accumulator.
+//
+// Two passes.  The row normalisers lse come first (the caller's, or the row-normaliser
+// kernel's).  Then attn_fwd_kernel forms, per (query tile of 128 rows, head), the exact
+// probabilities P = exp(scale q.k - lse) of each causal key tile, with no running
+// rescale, on the tensor cores:
+//   S   = Q K^T       tcgen05.mma, M = N = 128, K = 16 x 8 steps over d = 128, into TMEM
+//   P   = 2^(S scale log2e - lse log2e)   epilogue, written back to TMEM as bf16
+//   O  += P V         tcgen05.mma with A = P from TMEM, B = the key tile of V^T
+// and the column sums of P over the tile's 128 query rows (a warp reduce-scatter, then the
+// four TMEM lane quarters in order) go to a partial buffer, one slot per (prompt, head,
+// query tile, key tile).  imp_fwd_reduce_kernel adds a key's slots in a fixed order into
+// the accumulator: no floating-point atomics, repeated calls give identical bits.
+//
+// V enters the second MMA as its transpose V^T [Hkv][d][positions], written by
+// vt_transpose_kernel, so that it is K-major (keys contiguous) like every other operand;
+// each prompt starts at a multiple of 128 positions, which keeps every TMA coordinate
+// 16-byte aligned, and the padding is zero.
+//
+// attn_fwd_kernel: one persistent CTA per SM, 320 threads.
+//   warp 0      TMA producer (claims items, stages Q, and K + V^T per key tile, 2 stages)
+//   warp 1      MMA issuer: S(s) then O += P(s - 1) V(s - 1), so that the epilogue of one
+//               tile overlaps the MMAs of the next
+//   warps 2-9   epilogue: warp w reads TMEM lanes 32 (w % 4) .. (one query row each) and
+//               one 64-column half; P, the column sums, and O at the end of the item
+// TMEM: S double-buffered (2 x 128 columns), O (128), P double-buffered (2 x 64 columns of
+// bf16 pairs): all 512.  Every mbarrier wait is bounded; on expiry the CTA records
+// ESTP_ERR_TIMEOUT and drains.
+#include "importance_tc.cuh"
+#include "tcgen05.cuh"
+
+namespace estp {
+namespace {
+
+constexpr int kT = 128;                     // rows of a query or key tile
+constexpr int kD = 128;                     // head dim of this path
+constexpr int kAtomBytes = kT * 128;        // 128 rows x 64 bf16
+constexpr int kTileBytes = 2 * kAtomBytes;  // 128 rows x 128 bf16
+constexpr int kEpiWarp0 = 2, kEpiWarps = 8;
+constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
+constexpr int kSched = 4;
+// dynamic shared memory (offsets from a 1024-aligned base)
+constexpr int kQOff = 0;                          // [2] Q tiles
+constexpr int kRingOff = 2 * kTileBytes;          // [2 stages] K tile, then V^T tile
+constexpr int kCsOff = kRingOff + 4 * kTileBytes; // [2][4 quarters][128] column sums
+constexpr int kBarOff = kCsOff + 2 * 4 * kT * 4;
+constexpr int kNumBars = 16 + 3 + 4 + 2 * kSched;
+constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem address, abort flag, sched items
+constexpr int kSmemBytes = kMiscOff + 16 + 4 * kSched + 1024;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+// TMEM columns
+constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
+constexpr uint32_t kIdesc = idesc_bf16(kT, kT);   // M = N = 128 for both products
+
+struct FwdArgs {
+    const int32_t* cu;
+    const int32_t* base;    // items plan: prompt b's items start at base[b] (Hq per tile)
+    const int32_t* base2;   // partial slots: prompt b's start at base2[b] (Hq per tile pair)
+    PlanInfo* info;
+    const PlanInfo* info2;  // validity of the partial-slot plan
+    int B, Hq, Hkv;
+    int64_t sumT;
+    float scale_log2;
+    int exclude_self;
+    const float* lse;       // [Hq, sumT] natural log
+    __nv_bfloat16* O;       // [sumT, Hq, 128]
+    float* part;            // [slots][128]
+    int* status;
+};
+
+// A operand from TMEM: D (TMEM) = A (TMEM) B^T (+ D when acc != 0).
+__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(kIdesc), "r"(acc));
+}
+
+// 16 consecutive 32-bit TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // .x = lo (low half)
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ int64_t tri(int64_t n) { return n * (n + 1) / 2; }
+
+// Reduce-scatter over a warp: on entry lane l holds v[0..31] (32 columns), on exit v[0]
+// holds the warp sum of column l.  Every lane adds in the same order.
+__device__ __forceinline__ float warp_reduce_scatter32(float* v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int w = 16; w >= 1; w >>= 1) {
+        const bool upper = (lane & w) != 0;
+#pragma unroll
+        for (int j = 0; j < w; ++j) {
+            const float send = upper ? v[j] : v[j + w];
+            const float keep = upper ? v[j + w] : v[j];
+            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+        }
+    }
+    return v[0];
+}
+
+struct FwdItem {
+    int b, h, qt, nt, T;
+    int64_t t0;
+};
+
+__device__ __forceinline__ FwdItem fwd_item(const FwdArgs& a, int item) {
+    const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kT, a.Hq);
+    FwdItem t;
+    t.b = li.b;
+    t.h = li.hslot;
+    t.qt = li.qt;
+    t.t0 = li.t0;
+    t.T = li.T;
+    t.nt = (li.T + kT - 1) / kT;
+    return t;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                    const __grid_constant__ CUtensorMap tm_vt, const FwdArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+    float* cs = reinterpret_cast<float*>(sm + kCsOff);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kBarOff);
+    uint64_t* q_full = bars;           // [2]
+    uint64_t* q_empty = bars + 2;      // [2]
+    uint64_t* ring_full = bars + 4;    // [2]
+    uint64_t* ring_empty = bars + 6;   // [2]
+    uint64_t* s_full = bars + 8;       // [2]
+    uint64_t* s_empty = bars + 10;     // [2]
+    uint64_t* p_full = bars + 12;      // [2]
+    uint64_t* p_empty = bars + 14;     // [2]
+    uint64_t* o_full = bars + 16;
+    uint64_t* o_empty = bars + 17;
+    uint64_t* drain = bars + 18;
+    uint64_t* cs_full = bars + 19;     // [2] column sums of every quarter written
+    uint64_t* cs_empty = bars + 21;    // [2] column sums added up by the reader warps
+    uint64_t* sched_full = bars + 23;  // [kSched]
+    uint64_t* sched_empty = sched_full + kSched;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kMiscOff);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kMiscOff + 4);
+    volatile int* sched_item = reinterpret_cast<volatile int*>(sm + kMiscOff + 16);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&q_full[i], 1);
+            mbar_init(&q_empty[i], 1);
+            mbar_init(&ring_full[i], 1);
+            mbar_init(&ring_empty[i], 1);
+            mbar_init(&s_full[i], 1);
+            mbar_init(&s_empty[i], kEpiWarps);
+            mbar_init(&p_full[i], kEpiWarps);
+            mbar_init(&p_empty[i], 1);
+        }
+        mbar_init(o_full, 1);
+        mbar_init(o_empty, kEpiWarps);
+        mbar_init(drain, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&cs_full[i], kEpiWarps);
+            mbar_init(&cs_empty[i], kEpiWarps / 4);  // the quarter-0 warps, one per half
+        }
+        for (int i = 0; i < kSched; ++i) {
+            mbar_init(&sched_full[i], 1);
+            mbar_init(&sched_empty[i], 1 + kEpiWarps);  // MMA thread + epilogue warps
+        }
+        *abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(512));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    // the plans (and the lse values) are complete past this point
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int total = a.info->ok && a.info2->ok ? a.info->total : 0;
+
+    auto consume_item = [&](int k, bool warp_uniform) -> int {
+        const int slot = k % kSched;
+        const uint32_t par = (uint32_t)((k / kSched) & 1);
+        bool got;
+        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
+        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
+        if (!got) return -1;
+        const int item = sched_item[slot];
+        if (warp_uniform) __syncwarp();
+        if (!warp_uniform || lane == 0) mbar_arrive(&sched_empty[slot]);
+        return item;
+    };
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_q)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_vt)) : "memory");
+            uint32_t step = 0;
+            int n_items = 0;
+            int item = blockIdx.x;
+            for (int it = 0;; ++it) {
+                if (item >= total) item = -1;
+                const int slot = it % kSched;
+                if (it >= kSched &&
+                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
+                    break;
+                sched_item[slot] = item;
+                mbar_arrive(&sched_full[slot]);
+                if (item < 0) break;
+                const FwdItem t = fwd_item(a, item);
+                const int g = t.h / (a.Hq / a.Hkv);
+                const int fb = it & 1;
+                if (it >= 2 && !wait_bar(&q_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
+                mbar_expect_tx(&q_full[fb], kTileBytes);
+                for (int at = 0; at < 2; ++at)
+                    tma_load_3d(sm + kQOff + fb * kTileBytes + at * kAtomBytes, &tm_q, at * 64, t.h,
+                                (int)(t.t0 + t.qt * kT), &q_full[fb]);
+                ++n_items;
+                const int pstart = (a.base[t.b] / a.Hq) * kT;  // the prompt's first V^T position
+                bool ok = true;
+                for (int kt = 0; kt <= t.qt; ++kt, ++step) {
+                    const int stage = (int)(step & 1);
+                    const uint32_t u = step >> 1;
+                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* st = sm + kRingOff + stage * 2 * kTileBytes;
+                    mbar_expect_tx(&ring_full[stage], 2 * kTileBytes);
+                    for (int at = 0; at < 2; ++at) {
+                        tma_load_3d(st + at * kAtomBytes, &tm_k, at * 64, g, (int)(t.t0 + kt * kT),
+                                    &ring_full[stage]);
+                        tma_load_3d(st + kTileBytes + at * kAtomBytes, &tm_vt, pstart + kt * kT + at * 64,
+                                    0, g, &ring_full[stage]);
+                    }
+                }
+                if (!ok) break;
+                item = (int)gridDim.x + atomicAdd(&a.info->next, 1);
+            }
+            for (uint32_t i = 0; i < 2 && i < step; ++i)
+                drain_wait(&ring_full[(step - 1 - i) & 1], ((step - 1 - i) >> 1) & 1, a.status);
+            for (int fb = 0; fb < 2 && fb < n_items; ++fb)
+                drain_wait(&q_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------- MMA issuer
+        // One stream of steps across items: S(s) is issued before O += P(s - 1) V(s - 1),
+        // also when step s - 1 ended the previous item, so the tensor pipe computes the
+        // next item's first scores while the epilogue finishes the last tile of the one
+        // before.
+        if (lane == 0) {
+            struct Pending {
+                uint32_t step;
+                int it, fb;
+                bool first, last;
+            };
+            Pending prev{0, 0, 0, false, false};
+            bool have_prev = false, issued = false, ok = true;
+            // O += P(p) V(p): P from TMEM, V^T's key tile from the ring; after the item's
+            // last tile, O and the item's Q buffer are released
+            auto pv = [&](const Pending& p) -> bool {
+                const int pb = (int)(p.step & 1);
+                if (!wait_bar(&p_full[pb], (p.step >> 1) & 1, abort_flag, a.status)) return false;
+                if (p.first && p.it >= 1 && !wait_bar(o_empty, (p.it - 1) & 1, abort_flag, a.status))
+                    return false;
+                tc_fence_after();
+                const uint32_t va = smem_u32(sm + kRingOff + pb * 2 * kTileBytes + kTileBytes);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)
+                    mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
+                           sw128_desc(va + (kk >> 2) * kAtomBytes + (kk & 3) * 32),
+                           (p.first && kk == 0) ? 0u : 1u);
+                mma_commit(&ring_empty[pb]);
+                mma_commit(&p_empty[pb]);
+                if (p.last) {
+                    mma_commit(o_full);
+                    mma_commit(&q_empty[p.fb]);
+                }
+                return true;
+            };
+            uint32_t step = 0;
+            for (int it = 0; ok; ++it) {
+                const int item = consume_item(it, false);
+                if (item < 0) break;
+                const FwdItem t = fwd_item(a, item);
+                const int fb = it & 1;
+                if (!wait_bar(&q_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
+                const uint32_t qa = smem_u32(sm + kQOff + fb * kTileBytes);
+                for (int kt = 0; kt <= t.qt; ++kt, ++step) {
+                    const int stage = (int)(step & 1);
+                    const uint32_t u = step >> 1;
+                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status) ||
+                        (u >= 1 && !wait_bar(&s_empty[stage], (u - 1) & 1, abort_flag, a.status))) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    issued = true;
+                    const uint32_t ka = smem_u32(sm + kRingOff + stage * 2 * kTileBytes);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const uint32_t off = (uint32_t)((kk >> 2) * kAtomBytes + (kk & 3) * 32);
+                        mma_bf16<kIdesc>(tmem + kColS + stage * 128, sw128_desc(qa + off),
+                                         sw128_desc(ka + off), kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(&s_full[stage]);
+                    if (have_prev && !pv(prev)) {
+                        ok = false;
+                        break;
+                    }
+                    prev = Pending{step, it, fb, kt == 0, kt == t.qt};
+                    have_prev = true;
+                }
+            }
+            if (ok && have_prev) pv(prev);
+            if (issued) {
+                mma_commit(drain);
+                drain_wait(drain, 0, a.status);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------- epilogue
+        const int e = warp - kEpiWarp0;
+        const int q = warp & 3;                // TMEM lane quarter
+        const int half = e >> 2;               // 64-column half of S / P and of O's columns
+        const int row = q * 32 + lane;         // query row of the tile owned by this thread
+        const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+        uint32_t step = 0;
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            const int item = consume_item(it, true);
+            if (item < 0) break;
+            const FwdItem t = fwd_item(a, item);
+            const int i_loc = t.qt * kT + row;                 // query index in the prompt
+            const bool valid = i_loc < t.T;
+            const float lrow = valid ? a.lse[(int64_t)t.h * a.sumT + t.t0 + i_loc] * kLog2e : 0.f;
+            const int64_t slot0 = a.base2[t.b] + (int64_t)t.h * tri(t.nt) + tri(t.qt);
+            for (int kt = 0; kt <= t.qt; ++kt, ++step) {
+                const int sb = (int)(step & 1);
+                if (!warp_wait(&s_full[sb], (step >> 1) & 1, abort_flag, a.status) ||
+                    (step >= 2 && !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status))) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                float* csb = cs + sb * 4 * kT;
+                // the reader warps are done with this buffer's sums of step - 2
+                if (step >= 2 && !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch) {
+                    const int col0 = half * 64 + ch * 32;  // key column of v[0] in the tile
+                    float v[32];
+                    tmem_ld32(lane_base + kColS + sb * 128 + col0, v);
+                    tmem_wait_ld();
+                    if (ch == 1) {  // S of this warp read: the buffer may take the next tile
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&s_empty[sb]);
+                    }
+                    float c32[32];
+                    uint32_t w[16];
+#pragma unroll
+                    for (int c = 0; c < 32; c += 2) {
+                        const int j0 = kt * kT + col0 + c, j1 = j0 + 1;  // key indices in the prompt
+                        const float p0 = valid && j0 <= i_loc ? ex2(fmaf(v[c], a.scale_log2, -lrow)) : 0.f;
+                        const float p1 = valid && j1 <= i_loc ? ex2(fmaf(v[c + 1], a.scale_log2, -lrow)) : 0.f;
+                        w[c >> 1] = pack_bf16(p0, p1);
+                        c32[c] = a.exclude_self && j0 == i_loc ? 0.f : p0;
+                        c32[c + 1] = a.exclude_self && j1 == i_loc ? 0.f : p1;
+                    }
+                    tmem_st16(lane_base + kColP + sb * 64 + col0 / 2, w);
+                    csb[q * kT + col0 + lane] = warp_reduce_scatter32(c32);
+                }
+                asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&p_full[sb]);
+                    mbar_arrive(&cs_full[sb]);
+                }
+                if (q == 0) {  // the four quarters in order, two columns per lane
+                    if (!warp_wait(&cs_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const int c0 = half * 64 + 2 * lane;
+                    float2 sum;
+                    sum.x = (csb[c0] + csb[kT + c0]) + (csb[2 * kT + c0] + csb[3 * kT + c0]);
+                    sum.y = (csb[c0 + 1] + csb[kT + c0 + 1]) + (csb[2 * kT + c0 + 1] + csb[3 * kT + c0 + 1]);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&cs_empty[sb]);
+                    *reinterpret_cast<float2*>(a.part + (slot0 + kt) * kT + c0) = sum;
+                }
+            }
+            if (!ok) break;
+            // O of the item: this warp's 32 rows x 64 columns
+            if (!warp_wait(o_full, it & 1, abort_flag, a.status)) break;
+            tc_fence_after();
+#pragma unroll
+            for (int ch = 0; ch < 2; ++ch) {
+                float v[32];
+                tmem_ld32(lane_base + kColO + half * 64 + ch * 32, v);
+                tmem_wait_ld();
+                if (valid) {
+                    uint4* out = reinterpret_cast<uint4*>(
+                        a.O + ((t.t0 + i_loc) * a.Hq + t.h) * (int64_t)kD + half * 64 + ch * 32);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        out[k] = make_uint4(pack_bf16(v[8 * k], v[8 * k + 1]), pack_bf16(v[8 * k + 2], v[8 * k + 3]),
+                                            pack_bf16(v[8 * k + 4], v[8 * k + 5]), pack_bf16(v[8 * k + 6], v[8 * k + 7]));
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(o_empty);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) {
+        __syncwarp();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512));
+    }
+}
+
+// V [sumT, Hkv, 128] -> V^T [Hkv][128][L], prompt b's tokens at positions pstart_b ..,
+// pstart_b = 128 * (tiles of the prompts before b); the padding after each prompt is zero.
+// Block (32 positions, 32 rows of d) through a padded shared tile.
+__global__ void vt_transpose_kernel(const __nv_bfloat16* __restrict__ V, const int32_t* cu,
+                                    const int32_t* base, int B, int Hq, int Hkv, int64_t L,
+                                    __nv_bfloat16* __restrict__ Vt) {
+    __shared__ __nv_bfloat16 tile[32][33];
+    const int g = blockIdx.z;
+    const int64_t p0 = (int64_t)blockIdx.x * 32;
+    const int d0 = blockIdx.y * 32;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int32_t n_tiles = base[B] / Hq;
+    for (int r = ty; r < 32; r += blockDim.y) {  // r: position p0 + r, tx: d0 + tx
+        const int64_t p = p0 + r;
+        __nv_bfloat16 val = __float2bfloat16(0.f);
+        if (p < (int64_t)n_tiles * kT) {
+            const int b = upper_slot(base, B, (int)(p / kT) * Hq);
+            const int64_t tl = p - (int64_t)(base[b] / Hq) * kT;
+            if (tl < cu[b + 1] - cu[b]) val = V[((cu[b] + tl) * Hkv + g) * (int64_t)kD + d0 + tx];
+        }
+        tile[r][tx] = val;
+    }
+    __syncthreads();
+    for (int r = ty; r < 32; r += blockDim.y) {  // r: d0 + r, tx: position p0 + tx
+        const int64_t p = p0 + tx;
+        if (p < L) Vt[((int64_t)g * kD + d0 + r) * L + p] = tile[tx][r];
+    }
+}
+
+// C_j (+)= sum over heads h and query tiles qt >= kt(j) of the partial slots of key j, in
+// that fixed order.
+__global__ void imp_fwd_reduce_kernel(const float* __restrict__ part, const int32_t* cu,
+                                      const int32_t* base2, const PlanInfo* info, const PlanInfo* info2,
+                                      int B, int Hq,
+                                      int64_t sumT, int accumulate, float* acc) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= sumT) return;
+    float v = 0.f;
+    if (info->ok && info2->ok) {
+        const int b = upper_slot(cu, B, j);
+        const int T = cu[b + 1] - cu[b];
+        const int nt = (T + kT - 1) / kT;
+        const int jl = (int)(j - cu[b]), kt = jl / kT, col = jl - kt * kT;
+        for (int h = 0; h < Hq; ++h) {
+            const int64_t s0 = base2[b] + (int64_t)h * tri(nt);
+            constexpr int kBatch = 16;  // loads in flight before they are added, in order
+            for (int q0 = kt; q0 < nt; q0 += kBatch) {
+                float pv[kBatch];
+#pragma unroll
+                for (int i = 0; i < kBatch; ++i)
+                    pv[i] = q0 + i < nt ? part[(s0 + tri(q0 + i) + kt) * kT + col] : 0.f;
+#pragma unroll
+                for (int i = 0; i < kBatch; ++i)
+                    if (q0 + i < nt) v += pv[i];
+            }
+        }
+    }
+    acc[j] = accumulate ? acc[j] + v : v;
+}
+
+// bf16 tensor map of 3 dimensions (d0 innermost), box b0 x b1 x b2, 128-byte swizzle.
+estp_status make_map3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                      uint64_t s1, uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2) {
+    auto fn = tensor_map_encoder();
+    if (!fn) return fail(ESTP_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[3] = {d0, d1, d2};
+    cuuint64_t strides[2] = {s1, s2};
+    cuuint32_t box[3] = {b0, b1, b2};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                    box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(ESTP_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return ESTP_OK;
+}
+
+}  // namespace
+
+estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, const void* V,
+                                const float* lse_in, int Hq, int Hkv, float scale,
+                                const int32_t* cu, int B, int64_t sumT, int max_seqlen,
+                                bool exclude_self, bool accumulate, float* acc, void* O,
+                                cudaStream_t st) {
+    // workspace: V^T | partial slots | lse (when not given) | plans | row-normaliser plan
+    const int64_t max_nt = (max_seqlen + kT - 1) / kT;
+    const int64_t tiles_bound = (sumT + kT - 1) / kT + B;          // sum of nt_b
+    const int64_t L = tiles_bound * kT;                             // V^T positions
+    const int64_t slots_bound = (int64_t)Hq * tiles_bound * (max_nt + 1) / 2 + Hq;
+    const size_t off_part = align_up(sizeof(__nv_bfloat16) * (size_t)Hkv * kD * (size_t)L, 256);
+    const size_t off_lse = off_part + align_up(sizeof(float) * (size_t)slots_bound * kT, 256);
+    const size_t off_plan = off_lse + (lse_in ? 0 : align_up(sizeof(float) * (size_t)Hq * sumT, 256));
+    const size_t off_base2 = off_plan + align_up(sizeof(int32_t) * (size_t)(B + 1), 256);
+    const size_t off_info = off_base2 + align_up(sizeof(int32_t) * (size_t)(B + 1), 256);
+    const size_t off_info2 = off_info + 256;
+    const size_t off_lse_plan = off_info2 + 256;
+    // the row-normaliser kernel's own plan comes after ours: reserve for it too
+    estp_status s = ws_reserve(ctx, off_lse_plan + align_up(sizeof(int32_t) * (size_t)(B + 1), 256) +
+                                        sizeof(PlanInfo) + 256);
+    if (s != ESTP_OK) return s;
+    char* ws = static_cast<char*>(ctx->ws);
+    __nv_bfloat16* Vt = reinterpret_cast<__nv_bfloat16*>(ws);
+    float* part = reinterpret_cast<float*>(ws + off_part);
+    int32_t* base = reinterpret_cast<int32_t*>(ws + off_plan);
+    int32_t* base2 = reinterpret_cast<int32_t*>(ws + off_base2);
+    PlanInfo* info = reinterpret_cast<PlanInfo*>(ws + off_info);
+    PlanInfo* info2 = reinterpret_cast<PlanInfo*>(ws + off_info2);
+    const float* lse = lse_in;
+    if (!lse_in) {  // pass 1: the row normalisers of every head
+        float* l = reinterpret_cast<float*>(ws + off_lse);
+        ImpHeads all;
+        if ((s = build_heads(nullptr, Hq, Hq, Hkv, &all)) != ESTP_OK) return s;
+        if ((s = launch_lse_tc(ctx, Q, K, Hq, Hkv, kD, scale, all, cu, B, sumT, max_seqlen, l, st,
+                               off_lse_plan)) != ESTP_OK)
+            return s;
+        lse = l;
+    }
+    // plans: items (prompt, query tile, head), and the partial slots (tile pairs x heads)
+    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, ctx->status);
+    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 2, base2, info2, ctx->status);
+    const dim3 tgrid((unsigned)(L / 32), kD / 32, (unsigned)Hkv);
+    vt_transpose_kernel<<<tgrid, dim3(32, 8), 0, st>>>(static_cast<const __nv_bfloat16*>(V), cu, base, B,
+                                                       Hq, Hkv, L, Vt);
+    CUtensorMap mq, mk, mvt;
+    // Q, K: (d, head, token), one head's 64 x 128 atom per box; V^T: (position, d, head)
+    if ((s = make_map3(&mq, Q, kD, Hq, sumT, (uint64_t)kD * 2, (uint64_t)Hq * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
+    if ((s = make_map3(&mk, K, kD, Hkv, sumT, (uint64_t)kD * 2, (uint64_t)Hkv * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
+    if ((s = make_map3(&mvt, Vt, L, kD, Hkv, (uint64_t)L * 2, (uint64_t)L * kD * 2, 64, kD, 1)) != ESTP_OK) return s;
+    FwdArgs a{};
+    a.cu = cu; a.base = base; a.base2 = base2; a.info = info; a.info2 = info2;
+    a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.sumT = sumT;
+    a.scale_log2 = scale * kLog2e;
+    a.exclude_self = exclude_self ? 1 : 0;
+    a.lse = lse; a.O = static_cast<__nv_bfloat16*>(O); a.part = part; a.status = ctx->status;
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return cuda_fail(e, "attention forward smem attribute");
+    attn_fwd_kernel<<<(unsigned)ctx->num_sms, kThreads, kSmemBytes, st>>>(mq, mk, mvt, a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "attention forward launch");
+    imp_fwd_reduce_kernel<<<(unsigned)((sumT + 255) / 256), 256, 0, st>>>(part, cu, base2, info, info2, B, Hq, sumT,
+                                                                         accumulate ? 1 : 0, acc);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "attention forward reduce launch");
+}
+
+}  // namespace estp

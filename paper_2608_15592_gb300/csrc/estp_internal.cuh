@@ -116,6 +116,10 @@ estp_status launch_mlp_head_loss(estp_ctx* ctx, const float* pooled, int B, int6
                                  float* loss, const estp_mlp_grads& g, cudaStream_t st);
 estp_status launch_misalignment(estp_ctx* ctx, const float* H, const float* S, const int32_t* cu,
                                 int B, int64_t sumT, int pct, int32_t* counts, cudaStream_t st);
+estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, const void* V,
+                                const float* lse, int Hq, int Hkv, float scale, const int32_t* cu,
+                                int B, int64_t sumT, int max_seqlen, bool exclude_self,
+                                bool accumulate, float* acc, void* O, cudaStream_t st);
 estp_status launch_importance_finalize(estp_ctx* ctx, const float* acc, const int32_t* cu, int B,
                                        int64_t sumT, int n_layers, int n_heads, uint32_t flags,
                                        float* out, cudaStream_t st);

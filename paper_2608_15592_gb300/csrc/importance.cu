@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
         const int32_t len = cu[b + 1] - cu[b];
         if (len < 0 || len > max_seqlen) { bad = 1; continue; }
         const int nt = (len + tile - 1) / tile;
-        local += (int64_t)mult * (kind == 0 ? items_f(nt, qc) : nt);
+        local += (int64_t)mult * plan_count(nt, qc, kind);
     }
     int64_t inc = local;  // inclusive scan within the warp
 #pragma unroll
@@ -62,7 +62,7 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
         base[b] = ok ? (int32_t)run : 0;
         const int32_t len = cu[b + 1] - cu[b];
         const int nt = (len + tile - 1) / tile;
-        if (len >= 0) run += (int64_t)mult * (kind == 0 ? items_f(nt, qc) : nt);
+        if (len >= 0) run += (int64_t)mult * plan_count(nt, qc, kind);
     }
     if (tid == 1023) {
         base[B] = ok ? (int32_t)total : 0;

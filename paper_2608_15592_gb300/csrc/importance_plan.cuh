@@ -28,8 +28,14 @@ struct PlanInfo {
     int32_t pad;
 };
 
-// Prefix of per-prompt item counts (base[B+1]) and validation.  One CTA of 1024.
-// kind 0: importance items, n_groups * f(nt); kind 1: LSE items, n_heads * nt.
+// Per-prompt count of a plan of kind 0: importance items f(nt); kind 1: one per tile, nt;
+// kind 2: one per pair of tiles (query tile, key tile <= query tile), nt (nt + 1) / 2.
+__host__ __device__ __forceinline__ int64_t plan_count(int64_t nt, int qc, int kind) {
+    return kind == 0 ? items_f(nt, qc) : kind == 1 ? nt : nt * (nt + 1) / 2;
+}
+
+// Prefix of per-prompt counts (base[B+1]) and validation.  One CTA of 1024.
+// Each prompt counts mult * plan_count(nt, qc, kind).
 __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int B, int64_t sumT,
                                                          int max_seqlen, int tile, int qc,
                                                          int mult, int kind, int32_t* base,

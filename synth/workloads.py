@@ -23,6 +23,7 @@ S_LOGIT_ROWS = 3
 S_HIDDEN = 4
 S_HEAD_W = 5
 S_Q0 = 1000  # Q of layer l: S_Q0 + 2l, K of layer l: S_Q0 + 2l + 1
+S_V0 = 3000  # V of layer l: S_V0 + l
 
 
 @dataclass(frozen=True)
@@ -80,6 +81,9 @@ class Workload:
 
     def key_k(self, layer: int) -> int:
         return self.key(S_Q0 + 2 * layer + 1)
+
+    def key_v(self, layer: int) -> int:
+        return self.key(S_V0 + layer)
 
     # ------------------------------------------------------- head params
     def head_params(self):
