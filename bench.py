@@ -310,6 +310,7 @@ def run_ours(args, rank, world, local_rank):
     head_loss = time_head_loss(st, dev)
     misalign = time_misalignment(st)
     lm_head = time_lm_head(st, bf16_sus)
+    attn_fwd = time_attn_forward(st, bf16_sus, kern_ms)
     e2e_hidden = run_e2e_from_hidden(args, st, dev, world)
     clocks = clk.summary()
     del st
@@ -329,7 +330,7 @@ def run_ours(args, rank, world, local_rank):
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": st_launches(w) * K, "clocks": clocks,
         "head_loss": head_loss, "misalignment": misalign, "lm_head_entropy": lm_head,
-        "e2e_from_hidden": e2e_hidden,
+        "e2e_from_hidden": e2e_hidden, "attn_forward_importance": attn_fwd,
     }
 
 
@@ -415,6 +416,86 @@ def time_lm_head(st, peak_tflops, iters: int = 20, warmup: int = 30):
             "bound": "tensor", "achieved": tf, "unit": "TFLOP/s", "peak": peak_tflops,
             "frac": tf / peak_tflops, "tokens_per_s": st.sumT / (ms / 1e3),
             "logit_bytes_not_stored": 2 * st.sumT * w.V}
+
+
+def time_attn_forward(st, peak_tflops, kern_ms, iters: int = 20, warmup_s: float = 0.5):
+    """The prefill's attention forward with the importance column sums of the same
+    probabilities (estp_attn_forward_importance), one call per layer of the step, with
+    seeded V [sumT, Hkv, d]: not part of the step, which takes Q and K only; timed on its
+    own with CUDA events, with the row normalisers supplied (as a prefill provides them)
+    and computed by the call. Algorithmic work: the causal pairs of every head, 2 d flops
+    each for QK^T and for PV. For context, the same layer through torch's
+    scaled_dot_product_attention (one causal call per prompt; no importance)."""
+    import torch
+    import synth
+    from synth import device as sd
+    w = st.w
+    if w.dtype != "bf16" or w.d != 128:
+        return None
+    alg = algorithmic(w, st.cu_h)["lse"]["flops"] * 2
+    V = [sd.normal(w.key_v(layer), (st.sumT, w.Hkv, w.d), synth.BF16, device=st.Q[0].device)
+         for layer in w.layers]
+    O = torch.empty(st.sumT, w.Hq, w.d, dtype=torch.bfloat16, device=V[0].device)
+    n_layers = len(w.layers)
+    c = st.ctx
+
+    def fused(lse_given):
+        for n in range(n_layers):
+            if lse_given:
+                c.attn_lse(st.Q[n], st.K[n], st.cu, st.maxT, out=st.lse)
+            c.attn_forward_importance(st.Q[n], st.K[n], V[n], st.cu, st.maxT,
+                                      lse=st.lse if lse_given else None, accumulate=n > 0,
+                                      out=O)
+
+    def timed(fn, evs=None):
+        t_end = time.time() + warmup_s
+        while time.time() < t_end:
+            fn()
+            torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(iters):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        c.sync_status()
+        return a.elapsed_time(b) / (iters * n_layers)
+
+    # the fused call alone, its row normalisers precomputed once per layer
+    lse = [c.attn_lse(st.Q[n], st.K[n], st.cu, st.maxT) for n in range(n_layers)]
+
+    def fused_only():
+        for n in range(n_layers):
+            c.attn_forward_importance(st.Q[n], st.K[n], V[n], st.cu, st.maxT, lse=lse[n],
+                                      accumulate=n > 0, out=O)
+
+    ms_fused = timed(fused_only)
+    ms_internal = timed(lambda: fused(False))
+    tf = alg / (ms_fused / 1e3) / 1e12
+    out = {"ms_per_layer": ms_fused, "ms_per_layer_with_lse": ms_internal,
+           "layers": n_layers, "flops_per_layer": alg, "bound": "tensor", "achieved": tf,
+           "unit": "TFLOP/s", "peak": peak_tflops, "frac": tf / peak_tflops,
+           "launches_per_layer": 5, "unfused_importance_ms_per_layer":
+           kern_ms["lse"] + kern_ms["importance"]}
+    try:
+        import torch.nn.functional as F
+        bounds = [(int(st.cu_h[b]), int(st.cu_h[b + 1])) for b in range(w.B)]
+
+        def sdpa():
+            for n in range(n_layers):
+                for t0, t1 in bounds:
+                    if t1 > t0:
+                        q = st.Q[n][t0:t1].transpose(0, 1).unsqueeze(0)
+                        k = st.K[n][t0:t1].transpose(0, 1).unsqueeze(0)
+                        v = V[n][t0:t1].transpose(0, 1).unsqueeze(0)
+                        F.scaled_dot_product_attention(q, k, v, is_causal=True, enable_gqa=True)
+
+        out["torch_sdpa_ms_per_layer"] = timed(sdpa)
+    except Exception as exc:  # context only
+        out["torch_sdpa_ms_per_layer"] = None
+        out["torch_sdpa_error"] = str(exc)[:200]
+    del V, O
+    return out
 
 
 def time_misalignment(st, iters: int = 50):

@@ -20,11 +20,20 @@
 // 16-byte aligned, and the padding is zero.
 //
 // attn_fwd_kernel: one persistent CTA per SM, 320 threads.
-//   warp 0      TMA producer (claims items, stages Q, and K + V^T per key tile, 2 stages)
-//   warp 1      MMA issuer: S(s) then O += P(s - 1) V(s - 1), so that the epilogue of one
-//               tile overlaps the MMAs of the next
-//   warps 2-9   epilogue: warp w reads TMEM lanes 32 (w % 4) .. (one query row each) and
-//               one 64-column half; P, the column sums, and O at the end of the item
+//   warp 0      TMA producer: claims items, stages Q (2 buffers), K and V^T of each key
+//               tile (a ring of 2 each: a K tile is free once S is computed, a V^T tile
+//               once P V is)
+//   warp 1      issues S = Q K^T (as soon as a K tile and an S buffer are free)
+//   warp 2      issues O += P V (as soon as the epilogue has written P): two issuing
+//               threads, because one thread that issues 16 MMAs, makes 4 barrier checks
+//               and 5 commits per tile takes longer than the tensor pipe needs for them
+//   warps 3-18  epilogue, two groups of 8 that take the even and the odd key-tile steps
+//               (each S / P buffer belongs to one group); warp w reads TMEM lanes
+//               32 (w % 4) .. (one query row each) and one 64-column half: P, the column
+//               sums of its 32 rows, and O at the end of an item (by the group of its
+//               last step)
+//   warp 19     adds the four lane quarters' column sums of every tile, in order, and
+//               writes the tile's partial slot
 // TMEM: S double-buffered (2 x 128 columns), O (128), P double-buffered (2 x 64 columns of
 // bf16 pairs): all 512.  Every mbarrier wait is bounded; on expiry the CTA records
 // ESTP_ERR_TIMEOUT and drains.
@@ -38,18 +47,20 @@ constexpr int kT = 128;                     // rows of a query or key tile
 constexpr int kD = 128;                     // head dim of this path
 constexpr int kAtomBytes = kT * 128;        // 128 rows x 64 bf16
 constexpr int kTileBytes = 2 * kAtomBytes;  // 128 rows x 128 bf16
-constexpr int kEpiWarp0 = 2, kEpiWarps = 8;
-constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
+constexpr int kEpiWarp0 = 3, kEpiWarps = 16;
+constexpr int kGroupWarps = kEpiWarps / 2;        // warps of one epilogue group
+constexpr int kRedWarp = kEpiWarp0 + kEpiWarps;  // the column-sum reducer
+constexpr int kThreads = 32 * (kRedWarp + 1);
 constexpr int kSched = 4;
 // dynamic shared memory (offsets from a 1024-aligned base)
 constexpr int kQOff = 0;                          // [2] Q tiles
-constexpr int kRingOff = 2 * kTileBytes;          // [2 stages] K tile, then V^T tile
-constexpr int kCsOff = kRingOff + 4 * kTileBytes; // [2][4 quarters][128] column sums
+constexpr int kKOff = 2 * kTileBytes;             // [2 stages] K tiles
+constexpr int kVOff = 4 * kTileBytes;             // [2 stages] V^T tiles
+constexpr int kCsOff = 6 * kTileBytes;            // [2][4 quarters][128] column sums
 constexpr int kBarOff = kCsOff + 2 * 4 * kT * 4;
-constexpr int kNumBars = 16 + 3 + 4 + 2 * kSched;
-constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem address, abort flag, sched items
-constexpr int kSmemBytes = kMiscOff + 16 + 4 * kSched + 1024;
-static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+constexpr int kNumBars = 20 + 5 + 4 + 2 * kSched;
+constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem address, abort flag
+constexpr int kItemOff = kMiscOff + 16;           // [kSched] decoded items of the sched ring
 // TMEM columns
 constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdesc = idesc_bf16(kT, kT);   // M = N = 128 for both products
@@ -114,19 +125,28 @@ __device__ __forceinline__ float warp_reduce_scatter32(float* v) {
 }
 
 struct FwdItem {
-    int b, h, qt, nt, T;
+    int valid;              // 0: no more items
+    int h, qt, T;
     int64_t t0;
+    int64_t slot0;          // partial slot of (this head, query tile, key tile 0)
+    int pos0;               // V^T position of the prompt's first key
+    int pad;
 };
+constexpr int kSmemBytes = kItemOff + kSched * (int)sizeof(FwdItem) + 1024;
+static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
 __device__ __forceinline__ FwdItem fwd_item(const FwdArgs& a, int item) {
     const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kT, a.Hq);
     FwdItem t;
-    t.b = li.b;
+    t.valid = 1;
     t.h = li.hslot;
     t.qt = li.qt;
     t.t0 = li.t0;
     t.T = li.T;
-    t.nt = (li.T + kT - 1) / kT;
+    const int nt = (li.T + kT - 1) / kT;
+    t.slot0 = a.base2[li.b] + (int64_t)li.hslot * tri(nt) + tri(li.qt);
+    t.pos0 = (a.base[li.b] / a.Hq) * kT;
+    t.pad = 0;
     return t;
 }
 
@@ -140,45 +160,53 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kBarOff);
     uint64_t* q_full = bars;           // [2]
     uint64_t* q_empty = bars + 2;      // [2]
-    uint64_t* ring_full = bars + 4;    // [2]
-    uint64_t* ring_empty = bars + 6;   // [2]
-    uint64_t* s_full = bars + 8;       // [2]
-    uint64_t* s_empty = bars + 10;     // [2]
-    uint64_t* p_full = bars + 12;      // [2]
-    uint64_t* p_empty = bars + 14;     // [2]
-    uint64_t* o_full = bars + 16;
-    uint64_t* o_empty = bars + 17;
-    uint64_t* drain = bars + 18;
-    uint64_t* cs_full = bars + 19;     // [2] column sums of every quarter written
-    uint64_t* cs_empty = bars + 21;    // [2] column sums added up by the reader warps
-    uint64_t* sched_full = bars + 23;  // [kSched]
+    uint64_t* k_full = bars + 4;       // [2]
+    uint64_t* k_empty = bars + 6;      // [2]
+    uint64_t* v_full = bars + 8;       // [2]
+    uint64_t* v_empty = bars + 10;     // [2]
+    uint64_t* s_full = bars + 12;      // [2]
+    uint64_t* s_empty = bars + 14;     // [2]
+    uint64_t* p_full = bars + 16;      // [2]
+    uint64_t* p_empty = bars + 18;     // [2]
+    // [2] O complete, for the group that takes the parity of the item's last step: each
+    // group waits on every phase of its own barrier
+    uint64_t* o_full = bars + 20;
+    uint64_t* o_empty = bars + 22;
+    uint64_t* drain = bars + 23;       // [2] each issuer's MMAs done
+    uint64_t* cs_full = bars + 25;     // [2] column sums of every quarter written
+    uint64_t* cs_empty = bars + 27;    // [2] column sums added up by the reducer warp
+    uint64_t* sched_full = bars + 29;  // [kSched]
     uint64_t* sched_empty = sched_full + kSched;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kMiscOff + 4);
-    volatile int* sched_item = reinterpret_cast<volatile int*>(sm + kMiscOff + 16);
+    FwdItem* sched_item = reinterpret_cast<FwdItem*>(sm + kItemOff);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&q_full[i], 1);
             mbar_init(&q_empty[i], 1);
-            mbar_init(&ring_full[i], 1);
-            mbar_init(&ring_empty[i], 1);
+            mbar_init(&k_full[i], 1);
+            mbar_init(&k_empty[i], 1);
+            mbar_init(&v_full[i], 1);
+            mbar_init(&v_empty[i], 1);
             mbar_init(&s_full[i], 1);
-            mbar_init(&s_empty[i], kEpiWarps);
-            mbar_init(&p_full[i], kEpiWarps);
+            mbar_init(&s_empty[i], kGroupWarps);
+            mbar_init(&p_full[i], kGroupWarps);
             mbar_init(&p_empty[i], 1);
         }
-        mbar_init(o_full, 1);
-        mbar_init(o_empty, kEpiWarps);
-        mbar_init(drain, 1);
+        mbar_init(&o_full[0], 1);
+        mbar_init(&o_full[1], 1);
+        mbar_init(o_empty, kGroupWarps);
+        mbar_init(&drain[0], 1);
+        mbar_init(&drain[1], 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&cs_full[i], kEpiWarps);
-            mbar_init(&cs_empty[i], kEpiWarps / 4);  // the quarter-0 warps, one per half
+            mbar_init(&cs_full[i], kGroupWarps);
+            mbar_init(&cs_empty[i], 1);  // the reducer warp
         }
         for (int i = 0; i < kSched; ++i) {
             mbar_init(&sched_full[i], 1);
-            mbar_init(&sched_empty[i], 1 + kEpiWarps);  // MMA thread + epilogue warps
+            mbar_init(&sched_empty[i], 3 + kEpiWarps);  // issuers, epilogue and reducer warps
         }
         *abort_flag = 0;
         mbar_fence_init();
@@ -197,17 +225,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const int total = a.info->ok && a.info2->ok ? a.info->total : 0;
 
-    auto consume_item = [&](int k, bool warp_uniform) -> int {
+    // the k-th item of this CTA, decoded by the producer (valid = 0: no more items)
+    auto consume_item = [&](int k, bool warp_uniform) -> FwdItem {
         const int slot = k % kSched;
         const uint32_t par = (uint32_t)((k / kSched) & 1);
         bool got;
         if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
         else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
-        if (!got) return -1;
-        const int item = sched_item[slot];
+        FwdItem t{};
+        if (!got) return t;
+        t = sched_item[slot];
         if (warp_uniform) __syncwarp();
         if (!warp_uniform || lane == 0) mbar_arrive(&sched_empty[slot]);
-        return item;
+        return t;
     };
 
     if (warp == 0) {
@@ -216,19 +246,38 @@ __global__ void __launch_bounds__(kThreads, 1)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_q)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_vt)) : "memory");
-            uint32_t step = 0;
+            // V^T of step s is issued after K of step s + 1: it is needed one MMA pair
+            // later, and its ring slot frees later
+            struct VLoad {
+                int pos, g;
+                uint32_t step;
+            };
+            VLoad vp{0, 0, 0};
+            bool have_v = false, ok = true;
+            auto load_v = [&](const VLoad& v) -> bool {
+                const int stage = (int)(v.step & 1);
+                const uint32_t u = v.step >> 1;
+                if (u >= 1 && !wait_bar(&v_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
+                mbar_expect_tx(&v_full[stage], kTileBytes);
+                for (int at = 0; at < 2; ++at)
+                    tma_load_3d(sm + kVOff + stage * kTileBytes + at * kAtomBytes, &tm_vt,
+                                v.pos + at * 64, 0, v.g, &v_full[stage]);
+                return true;
+            };
+            uint32_t step = 0, v_issued = 0;
             int n_items = 0;
             int item = blockIdx.x;
-            for (int it = 0;; ++it) {
+            for (int it = 0; ok; ++it) {
                 if (item >= total) item = -1;
                 const int slot = it % kSched;
                 if (it >= kSched &&
                     !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
                     break;
-                sched_item[slot] = item;
+                FwdItem t{};
+                if (item >= 0) t = fwd_item(a, item);
+                sched_item[slot] = t;
                 mbar_arrive(&sched_full[slot]);
                 if (item < 0) break;
-                const FwdItem t = fwd_item(a, item);
                 const int g = t.h / (a.Hq / a.Hkv);
                 const int fb = it & 1;
                 if (it >= 2 && !wait_bar(&q_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
@@ -237,140 +286,166 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_3d(sm + kQOff + fb * kTileBytes + at * kAtomBytes, &tm_q, at * 64, t.h,
                                 (int)(t.t0 + t.qt * kT), &q_full[fb]);
                 ++n_items;
-                const int pstart = (a.base[t.b] / a.Hq) * kT;  // the prompt's first V^T position
-                bool ok = true;
+                const int pstart = t.pos0;
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int stage = (int)(step & 1);
                     const uint32_t u = step >> 1;
-                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                    if (u >= 1 && !wait_bar(&k_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
-                    uint8_t* st = sm + kRingOff + stage * 2 * kTileBytes;
-                    mbar_expect_tx(&ring_full[stage], 2 * kTileBytes);
-                    for (int at = 0; at < 2; ++at) {
-                        tma_load_3d(st + at * kAtomBytes, &tm_k, at * 64, g, (int)(t.t0 + kt * kT),
-                                    &ring_full[stage]);
-                        tma_load_3d(st + kTileBytes + at * kAtomBytes, &tm_vt, pstart + kt * kT + at * 64,
-                                    0, g, &ring_full[stage]);
+                    mbar_expect_tx(&k_full[stage], kTileBytes);
+                    for (int at = 0; at < 2; ++at)
+                        tma_load_3d(sm + kKOff + stage * kTileBytes + at * kAtomBytes, &tm_k, at * 64, g,
+                                    (int)(t.t0 + kt * kT), &k_full[stage]);
+                    if (have_v) {
+                        if (!load_v(vp)) {
+                            ok = false;
+                            break;
+                        }
+                        ++v_issued;
                     }
+                    vp = VLoad{pstart + kt * kT, g, step};
+                    have_v = true;
                 }
                 if (!ok) break;
                 item = (int)gridDim.x + atomicAdd(&a.info->next, 1);
             }
+            if (ok && have_v && load_v(vp)) ++v_issued;
+            // every copy in flight lands before the CTA exits
             for (uint32_t i = 0; i < 2 && i < step; ++i)
-                drain_wait(&ring_full[(step - 1 - i) & 1], ((step - 1 - i) >> 1) & 1, a.status);
+                drain_wait(&k_full[(step - 1 - i) & 1], ((step - 1 - i) >> 1) & 1, a.status);
+            for (uint32_t i = 0; i < 2 && i < v_issued; ++i)
+                drain_wait(&v_full[(v_issued - 1 - i) & 1], ((v_issued - 1 - i) >> 1) & 1, a.status);
             for (int fb = 0; fb < 2 && fb < n_items; ++fb)
                 drain_wait(&q_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
         }
     } else if (warp == 1) {
-        // ---------------------------------------------------------- MMA issuer
-        // One stream of steps across items: S(s) is issued before O += P(s - 1) V(s - 1),
-        // also when step s - 1 ended the previous item, so the tensor pipe computes the
-        // next item's first scores while the epilogue finishes the last tile of the one
-        // before.
+        // ------------------------------------------------------------ S issuer
         if (lane == 0) {
-            struct Pending {
-                uint32_t step;
-                int it, fb;
-                bool first, last;
-            };
-            Pending prev{0, 0, 0, false, false};
-            bool have_prev = false, issued = false, ok = true;
-            // O += P(p) V(p): P from TMEM, V^T's key tile from the ring; after the item's
-            // last tile, O and the item's Q buffer are released
-            auto pv = [&](const Pending& p) -> bool {
-                const int pb = (int)(p.step & 1);
-                if (!wait_bar(&p_full[pb], (p.step >> 1) & 1, abort_flag, a.status)) return false;
-                if (p.first && p.it >= 1 && !wait_bar(o_empty, (p.it - 1) & 1, abort_flag, a.status))
-                    return false;
-                tc_fence_after();
-                const uint32_t va = smem_u32(sm + kRingOff + pb * 2 * kTileBytes + kTileBytes);
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk)
-                    mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                           sw128_desc(va + (kk >> 2) * kAtomBytes + (kk & 3) * 32),
-                           (p.first && kk == 0) ? 0u : 1u);
-                mma_commit(&ring_empty[pb]);
-                mma_commit(&p_empty[pb]);
-                if (p.last) {
-                    mma_commit(o_full);
-                    mma_commit(&q_empty[p.fb]);
-                }
-                return true;
-            };
             uint32_t step = 0;
+            bool issued = false, ok = true;
             for (int it = 0; ok; ++it) {
-                const int item = consume_item(it, false);
-                if (item < 0) break;
-                const FwdItem t = fwd_item(a, item);
+                const FwdItem t = consume_item(it, false);
+                if (!t.valid) break;
                 const int fb = it & 1;
                 if (!wait_bar(&q_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
                 const uint32_t qa = smem_u32(sm + kQOff + fb * kTileBytes);
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int stage = (int)(step & 1);
                     const uint32_t u = step >> 1;
-                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status) ||
+                    if (!wait_bar(&k_full[stage], u & 1, abort_flag, a.status) ||
                         (u >= 1 && !wait_bar(&s_empty[stage], (u - 1) & 1, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     issued = true;
-                    const uint32_t ka = smem_u32(sm + kRingOff + stage * 2 * kTileBytes);
+                    const uint32_t ka = smem_u32(sm + kKOff + stage * kTileBytes);
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
                         const uint32_t off = (uint32_t)((kk >> 2) * kAtomBytes + (kk & 3) * 32);
                         mma_bf16<kIdesc>(tmem + kColS + stage * 128, sw128_desc(qa + off),
                                          sw128_desc(ka + off), kk > 0 ? 1u : 0u);
                     }
+                    mma_commit(&k_empty[stage]);
                     mma_commit(&s_full[stage]);
-                    if (have_prev && !pv(prev)) {
+                    if (kt == t.qt) mma_commit(&q_empty[fb]);  // the item's last use of Q
+                }
+            }
+            if (issued) {
+                mma_commit(&drain[0]);
+                drain_wait(&drain[0], 0, a.status);
+            }
+        }
+    } else if (warp == 2) {
+        // ----------------------------------------------------------- PV issuer
+        // O += P(s) V(s): P from TMEM, V^T's key tile from the ring; the first tile of an
+        // item overwrites O (once the epilogue has read the previous item's O), the last
+        // one hands O to the epilogue group that takes its parity
+        if (lane == 0) {
+            uint32_t step = 0;
+            bool issued = false, ok = true;
+            for (int it = 0; ok; ++it) {
+                const FwdItem t = consume_item(it, false);
+                if (!t.valid) break;
+                for (int kt = 0; kt <= t.qt; ++kt, ++step) {
+                    const int pb = (int)(step & 1);
+                    if (!wait_bar(&v_full[pb], (step >> 1) & 1, abort_flag, a.status) ||
+                        !wait_bar(&p_full[pb], (step >> 1) & 1, abort_flag, a.status) ||
+                        (kt == 0 && it >= 1 && !wait_bar(o_empty, (it - 1) & 1, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
-                    prev = Pending{step, it, fb, kt == 0, kt == t.qt};
-                    have_prev = true;
+                    tc_fence_after();
+                    issued = true;
+                    const uint32_t va = smem_u32(sm + kVOff + pb * kTileBytes);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk)
+                        mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
+                               sw128_desc(va + (kk >> 2) * kAtomBytes + (kk & 3) * 32),
+                               (kt == 0 && kk == 0) ? 0u : 1u);
+                    mma_commit(&v_empty[pb]);
+                    mma_commit(&p_empty[pb]);
+                    if (kt == t.qt) mma_commit(&o_full[pb]);
                 }
             }
-            if (ok && have_prev) pv(prev);
             if (issued) {
-                mma_commit(drain);
-                drain_wait(drain, 0, a.status);
+                mma_commit(&drain[1]);
+                drain_wait(&drain[1], 0, a.status);
+            }
+        }
+    } else if (warp == kRedWarp) {
+        // ------------------------------------------------------ column-sum reducer
+        // every tile of every item, in order: the sums of the four lane quarters, added
+        // in quarter order, 4 columns per lane, written as the tile's partial slot
+        uint32_t step = 0;
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            const FwdItem t = consume_item(it, true);
+            if (!t.valid) break;
+            for (int kt = 0; kt <= t.qt; ++kt, ++step) {
+                const int sb = (int)(step & 1);
+                if (!warp_wait(&cs_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                const float4* c4 = reinterpret_cast<const float4*>(cs + sb * 4 * kT) + lane;
+                const float4 x0 = c4[0], x1 = c4[kT / 4], x2 = c4[2 * kT / 4], x3 = c4[3 * kT / 4];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&cs_empty[sb]);
+                const float4 sum = make_float4((x0.x + x1.x) + (x2.x + x3.x), (x0.y + x1.y) + (x2.y + x3.y),
+                                               (x0.z + x1.z) + (x2.z + x3.z), (x0.w + x1.w) + (x2.w + x3.w));
+                reinterpret_cast<float4*>(a.part + (t.slot0 + kt) * kT)[lane] = sum;
             }
         }
     } else {
         // ------------------------------------------------------------- epilogue
         const int e = warp - kEpiWarp0;
         const int q = warp & 3;                // TMEM lane quarter
-        const int half = e >> 2;               // 64-column half of S / P and of O's columns
+        const int grp = (e >> 2) & 1;          // takes the steps of this parity
+        const int half = e >> 3;               // 64-column half of S / P and of O's columns
         const int row = q * 32 + lane;         // query row of the tile owned by this thread
         const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
-        uint32_t step = 0;
+        uint32_t step = 0, n_out = 0;  // n_out: items whose O this group has read
         bool ok = true;
         for (int it = 0; ok; ++it) {
-            const int item = consume_item(it, true);
-            if (item < 0) break;
-            const FwdItem t = fwd_item(a, item);
+            const FwdItem t = consume_item(it, true);
+            if (!t.valid) break;
             const int i_loc = t.qt * kT + row;                 // query index in the prompt
             const bool valid = i_loc < t.T;
-            const float lrow = valid ? a.lse[(int64_t)t.h * a.sumT + t.t0 + i_loc] * kLog2e : 0.f;
-            const int64_t slot0 = a.base2[t.b] + (int64_t)t.h * tri(t.nt) + tri(t.qt);
+            // a row past the prompt gets lse = +inf: its probabilities are exactly 0
+            const float lrow = valid ? a.lse[(int64_t)t.h * a.sumT + t.t0 + i_loc] * kLog2e : INFINITY;
             for (int kt = 0; kt <= t.qt; ++kt, ++step) {
-                const int sb = (int)(step & 1);
-                if (!warp_wait(&s_full[sb], (step >> 1) & 1, abort_flag, a.status) ||
-                    (step >= 2 && !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status))) {
+                if ((int)(step & 1) != grp) continue;
+                const int sb = grp;
+                if (!warp_wait(&s_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 float* csb = cs + sb * 4 * kT;
-                // the reader warps are done with this buffer's sums of step - 2
-                if (step >= 2 && !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
-                    ok = false;
-                    break;
-                }
-#pragma unroll
+#pragma unroll 1
                 for (int ch = 0; ch < 2; ++ch) {
                     const int col0 = half * 64 + ch * 32;  // key column of v[0] in the tile
                     float v[32];
@@ -381,20 +456,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&s_empty[sb]);
                     }
-                    float c32[32];
                     uint32_t w[16];
+                    if (kt == t.qt) {  // the diagonal tile: causal mask, and the self term
+                        const int d0 = col0 - row;  // key minus query index of v[0]
 #pragma unroll
-                    for (int c = 0; c < 32; c += 2) {
-                        const int j0 = kt * kT + col0 + c, j1 = j0 + 1;  // key indices in the prompt
-                        const float p0 = valid && j0 <= i_loc ? ex2(fmaf(v[c], a.scale_log2, -lrow)) : 0.f;
-                        const float p1 = valid && j1 <= i_loc ? ex2(fmaf(v[c + 1], a.scale_log2, -lrow)) : 0.f;
-                        w[c >> 1] = pack_bf16(p0, p1);
-                        c32[c] = a.exclude_self && j0 == i_loc ? 0.f : p0;
-                        c32[c + 1] = a.exclude_self && j1 == i_loc ? 0.f : p1;
+                        for (int c = 0; c < 32; ++c) v[c] = d0 + c <= 0 ? ex2(fmaf(v[c], a.scale_log2, -lrow)) : 0.f;
+#pragma unroll
+                        for (int c = 0; c < 32; c += 2) w[c >> 1] = pack_bf16(v[c], v[c + 1]);
+                        if (a.exclude_self) {
+#pragma unroll
+                            for (int c = 0; c < 32; ++c) v[c] = d0 + c == 0 ? 0.f : v[c];
+                        }
+                    } else {  // every key precedes every query of the tile
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) v[c] = ex2(fmaf(v[c], a.scale_log2, -lrow));
+#pragma unroll
+                        for (int c = 0; c < 32; c += 2) w[c >> 1] = pack_bf16(v[c], v[c + 1]);
+                    }
+                    // P V of step - 2 has read this P buffer, and the reader warps have
+                    // added up this buffer's column sums of step - 2
+                    if (ch == 0 && step >= 2 &&
+                        !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
                     }
                     tmem_st16(lane_base + kColP + sb * 64 + col0 / 2, w);
-                    csb[q * kT + col0 + lane] = warp_reduce_scatter32(c32);
+                    const float sum = warp_reduce_scatter32(v);
+                    if (ch == 0 && step >= 2 &&
+                        !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    csb[q * kT + col0 + lane] = sum;
                 }
+                if (!ok) break;
                 asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 tc_fence_before();
                 __syncwarp();
@@ -402,23 +497,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive(&p_full[sb]);
                     mbar_arrive(&cs_full[sb]);
                 }
-                if (q == 0) {  // the four quarters in order, two columns per lane
-                    if (!warp_wait(&cs_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
-                    const int c0 = half * 64 + 2 * lane;
-                    float2 sum;
-                    sum.x = (csb[c0] + csb[kT + c0]) + (csb[2 * kT + c0] + csb[3 * kT + c0]);
-                    sum.y = (csb[c0 + 1] + csb[kT + c0 + 1]) + (csb[2 * kT + c0 + 1] + csb[3 * kT + c0 + 1]);
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&cs_empty[sb]);
-                    *reinterpret_cast<float2*>(a.part + (slot0 + kt) * kT + c0) = sum;
-                }
             }
             if (!ok) break;
+            if ((int)((step - 1) & 1) != grp) continue;  // the other group ends this item
             // O of the item: this warp's 32 rows x 64 columns
-            if (!warp_wait(o_full, it & 1, abort_flag, a.status)) break;
+            if (!warp_wait(&o_full[grp], n_out & 1, abort_flag, a.status)) break;
+            ++n_out;
             tc_fence_after();
 #pragma unroll
             for (int ch = 0; ch < 2; ++ch) {
@@ -450,51 +534,63 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // V [sumT, Hkv, 128] -> V^T [Hkv][128][L], prompt b's tokens at positions pstart_b ..,
 // pstart_b = 128 * (tiles of the prompts before b); the padding after each prompt is zero.
-// Block (32 positions, 32 rows of d) through a padded shared tile.
-__global__ void vt_transpose_kernel(const __nv_bfloat16* __restrict__ V, const int32_t* cu,
-                                    const int32_t* base, int B, int Hq, int Hkv, int64_t L,
-                                    __nv_bfloat16* __restrict__ Vt) {
-    __shared__ __nv_bfloat16 tile[32][33];
-    const int g = blockIdx.z;
-    const int64_t p0 = (int64_t)blockIdx.x * 32;
-    const int d0 = blockIdx.y * 32;
-    const int tx = threadIdx.x, ty = threadIdx.y;
+// A block moves 64 positions (inside one prompt's 128-aligned span) x 128 d of one KV head
+// through shared memory, with 16-byte loads and stores on both sides.
+constexpr int kTrPos = 64;
+__global__ void __launch_bounds__(256) vt_transpose_kernel(const __nv_bfloat16* __restrict__ V,
+                                                           const int32_t* cu, const int32_t* base, int B,
+                                                           int Hq, int Hkv, int64_t L,
+                                                           __nv_bfloat16* __restrict__ Vt) {
+    __shared__ __align__(16) uint16_t tile[kTrPos][kD + 8];  // [position][d], rows padded by 16 bytes
+    const int g = blockIdx.y;
+    const int64_t p0 = (int64_t)blockIdx.x * kTrPos;
     const int32_t n_tiles = base[B] / Hq;
-    for (int r = ty; r < 32; r += blockDim.y) {  // r: position p0 + r, tx: d0 + tx
-        const int64_t p = p0 + r;
-        __nv_bfloat16 val = __float2bfloat16(0.f);
-        if (p < (int64_t)n_tiles * kT) {
-            const int b = upper_slot(base, B, (int)(p / kT) * Hq);
-            const int64_t tl = p - (int64_t)(base[b] / Hq) * kT;
-            if (tl < cu[b + 1] - cu[b]) val = V[((cu[b] + tl) * Hkv + g) * (int64_t)kD + d0 + tx];
-        }
-        tile[r][tx] = val;
+    int64_t src0 = 0, n_valid = 0;  // first source token of the block, tokens that exist
+    if (p0 < (int64_t)n_tiles * kT) {
+        const int b = upper_slot(base, B, (int)(p0 / kT) * Hq);
+        const int64_t tl0 = p0 - (int64_t)(base[b] / Hq) * kT;
+        src0 = cu[b] + tl0;
+        n_valid = min((int64_t)kTrPos, (int64_t)(cu[b + 1] - cu[b]) - tl0);
+    }
+    for (int c = threadIdx.x; c < kTrPos * (kD / 8); c += blockDim.x) {
+        const int r = c / (kD / 8), q = c % (kD / 8);  // position r, d values 8q .. 8q + 7
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (r < n_valid)
+            val = *reinterpret_cast<const uint4*>(V + ((src0 + r) * Hkv + g) * (int64_t)kD + q * 8);
+        *reinterpret_cast<uint4*>(&tile[r][q * 8]) = val;
     }
     __syncthreads();
-    for (int r = ty; r < 32; r += blockDim.y) {  // r: d0 + r, tx: position p0 + tx
-        const int64_t p = p0 + tx;
-        if (p < L) Vt[((int64_t)g * kD + d0 + r) * L + p] = tile[tx][r];
+    for (int c = threadIdx.x; c < kD * (kTrPos / 8); c += blockDim.x) {
+        const int dd = c / (kTrPos / 8), q = c % (kTrPos / 8);  // d row dd, positions 8q .. 8q + 7
+        uint32_t w[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            w[k] = (uint32_t)tile[q * 8 + 2 * k][dd] | ((uint32_t)tile[q * 8 + 2 * k + 1][dd] << 16);
+        *reinterpret_cast<uint4*>(Vt + ((int64_t)g * kD + dd) * L + p0 + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
-// C_j (+)= sum over heads h and query tiles qt >= kt(j) of the partial slots of key j, in
-// that fixed order.
-__global__ void imp_fwd_reduce_kernel(const float* __restrict__ part, const int32_t* cu,
-                                      const int32_t* base2, const PlanInfo* info, const PlanInfo* info2,
-                                      int B, int Hq,
-                                      int64_t sumT, int accumulate, float* acc) {
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= sumT) return;
+// C_j (+)= sum over heads h and query tiles qt >= kt(j) of the partial slots of key j.  A block
+// takes 32 keys; its warp w sums heads w, w + 8, .. (each over qt in order), and the 8 warp
+// sums are added in order: a fixed order, whatever the launch.
+constexpr int kRedHeadLanes = 8;
+__global__ void __launch_bounds__(32 * kRedHeadLanes)
+    imp_fwd_reduce_kernel(const float* __restrict__ part, const int32_t* cu, const int32_t* base2,
+                          const PlanInfo* info, const PlanInfo* info2, int B, int Hq, int64_t sumT,
+                          int accumulate, float* acc) {
+    __shared__ float red[kRedHeadLanes][32];
+    const int jj = threadIdx.x & 31, hl = threadIdx.x >> 5;
+    const int64_t j = (int64_t)blockIdx.x * 32 + jj;
     float v = 0.f;
-    if (info->ok && info2->ok) {
+    if (j < sumT && info->ok && info2->ok) {
         const int b = upper_slot(cu, B, j);
         const int T = cu[b + 1] - cu[b];
         const int nt = (T + kT - 1) / kT;
         const int jl = (int)(j - cu[b]), kt = jl / kT, col = jl - kt * kT;
-        for (int h = 0; h < Hq; ++h) {
+        for (int h = hl; h < Hq; h += kRedHeadLanes) {
             const int64_t s0 = base2[b] + (int64_t)h * tri(nt);
-            constexpr int kBatch = 16;  // loads in flight before they are added, in order
+            float vh = 0.f;
+            constexpr int kBatch = 8;  // loads in flight before they are added, in order
             for (int q0 = kt; q0 < nt; q0 += kBatch) {
                 float pv[kBatch];
 #pragma unroll
@@ -502,11 +598,19 @@ __global__ void imp_fwd_reduce_kernel(const float* __restrict__ part, const int3
                     pv[i] = q0 + i < nt ? part[(s0 + tri(q0 + i) + kt) * kT + col] : 0.f;
 #pragma unroll
                 for (int i = 0; i < kBatch; ++i)
-                    if (q0 + i < nt) v += pv[i];
+                    if (q0 + i < nt) vh += pv[i];
             }
+            v += vh;
         }
     }
-    acc[j] = accumulate ? acc[j] + v : v;
+    red[hl][jj] = v;
+    __syncthreads();
+    if (hl == 0 && j < sumT) {
+        float sum = 0.f;
+#pragma unroll
+        for (int k = 0; k < kRedHeadLanes; ++k) sum += red[k][jj];
+        acc[j] = accumulate ? acc[j] + sum : sum;
+    }
 }
 
 // bf16 tensor map of 3 dimensions (d0 innermost), box b0 x b1 x b2, 128-byte swizzle.
@@ -568,9 +672,8 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     // plans: items (prompt, query tile, head), and the partial slots (tile pairs x heads)
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, ctx->status);
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 2, base2, info2, ctx->status);
-    const dim3 tgrid((unsigned)(L / 32), kD / 32, (unsigned)Hkv);
-    vt_transpose_kernel<<<tgrid, dim3(32, 8), 0, st>>>(static_cast<const __nv_bfloat16*>(V), cu, base, B,
-                                                       Hq, Hkv, L, Vt);
+    vt_transpose_kernel<<<dim3((unsigned)(L / kTrPos), (unsigned)Hkv), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(V), cu, base, B, Hq, Hkv, L, Vt);
     CUtensorMap mq, mk, mvt;
     // Q, K: (d, head, token), one head's 64 x 128 atom per box; V^T: (position, d, head)
     if ((s = make_map3(&mq, Q, kD, Hq, sumT, (uint64_t)kD * 2, (uint64_t)Hq * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
@@ -587,8 +690,8 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     attn_fwd_kernel<<<(unsigned)ctx->num_sms, kThreads, kSmemBytes, st>>>(mq, mk, mvt, a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "attention forward launch");
-    imp_fwd_reduce_kernel<<<(unsigned)((sumT + 255) / 256), 256, 0, st>>>(part, cu, base2, info, info2, B, Hq, sumT,
-                                                                         accumulate ? 1 : 0, acc);
+    imp_fwd_reduce_kernel<<<(unsigned)((sumT + 31) / 32), 32 * kRedHeadLanes, 0, st>>>(
+        part, cu, base2, info, info2, B, Hq, sumT, accumulate ? 1 : 0, acc);
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "attention forward reduce launch");
 }
