@@ -90,13 +90,31 @@ __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_
         "r"(a_tmem), "l"(b), "r"(kIdesc), "r"(acc));
 }
 
-// 16 consecutive 32-bit TMEM columns of this thread's lane.
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+// tcgen05.ld .16x256b.x8: 16 lanes from the lane of taddr, 64 columns.  Thread t gets, for
+// k = 0..7, r[4k + 0..1] = lane t/4, columns 8k + 2 (t%4) + 0..1 and r[4k + 2..3] = the
+// same columns of lane t/4 + 8.
+__device__ __forceinline__ void tmem_ld16x256_x8(uint32_t taddr, uint32_t* r) {
     asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+        "%28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+}
+
+// tcgen05.st .16x128b.x8: 16 lanes from the lane of taddr, 32 columns.  Thread t writes,
+// for k = 0..7, w[2k] to lane t/4, column 4k + t%4, and w[2k + 1] to lane t/4 + 8.
+__device__ __forceinline__ void tmem_st16x128_x8(uint32_t taddr, const uint32_t* w) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x128b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
         "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7]),
+        "r"(w[8]), "r"(w[9]), "r"(w[10]), "r"(w[11]), "r"(w[12]), "r"(w[13]), "r"(w[14]), "r"(w[15])
         : "memory");
 }
 
@@ -106,23 +124,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 __device__ __forceinline__ int64_t tri(int64_t n) { return n * (n + 1) / 2; }
-
-// Reduce-scatter over a warp: on entry lane l holds v[0..31] (32 columns), on exit v[0]
-// holds the warp sum of column l.  Every lane adds in the same order.
-__device__ __forceinline__ float warp_reduce_scatter32(float* v) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int w = 16; w >= 1; w >>= 1) {
-        const bool upper = (lane & w) != 0;
-#pragma unroll
-        for (int j = 0; j < w; ++j) {
-            const float send = upper ? v[j] : v[j + w];
-            const float keep = upper ? v[j + w] : v[j];
-            v[j] = keep + __shfl_xor_sync(0xffffffffu, send, w);
-        }
-    }
-    return v[0];
-}
 
 struct FwdItem {
     int valid;              // 0: no more items
@@ -427,6 +428,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int half = e >> 3;               // 64-column half of S / P and of O's columns
         const int row = q * 32 + lane;         // query row of the tile owned by this thread
         const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+        // S / P layout (16x256b / 16x128b): thread (g, c) = (lane / 4, lane % 4) holds rows
+        // 32q + g + 8r, r = 0..3, and key columns 8k + 2c + 0..1, k = 0..7, of its half
+        const int g8 = lane >> 2, c4 = lane & 3;
         uint32_t step = 0, n_out = 0;  // n_out: items whose O this group has read
         bool ok = true;
         for (int it = 0; ok; ++it) {
@@ -434,8 +438,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!t.valid) break;
             const int i_loc = t.qt * kT + row;                 // query index in the prompt
             const bool valid = i_loc < t.T;
-            // a row past the prompt gets lse = +inf: its probabilities are exactly 0
-            const float lrow = valid ? a.lse[(int64_t)t.h * a.sumT + t.t0 + i_loc] * kLog2e : INFINITY;
+            // the row normalisers (log2 units) of the 4 rows of the S / P layout; a row past
+            // the prompt gets +inf, so its probabilities are exactly 0
+            float lr[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int ir = t.qt * kT + q * 32 + g8 + 8 * r;
+                lr[r] = ir < t.T ? a.lse[(int64_t)t.h * a.sumT + t.t0 + ir] * kLog2e : INFINITY;
+            }
             for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                 if ((int)(step & 1) != grp) continue;
                 const int sb = grp;
@@ -445,51 +455,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 float* csb = cs + sb * 4 * kT;
+                const bool diag = kt == t.qt;
+                float csum[16];  // column sums of this thread's rows: [2k + e] for column 8k + 2c4 + e
 #pragma unroll 1
-                for (int ch = 0; ch < 2; ++ch) {
-                    const int col0 = half * 64 + ch * 32;  // key column of v[0] in the tile
-                    float v[32];
-                    tmem_ld32(lane_base + kColS + sb * 128 + col0, v);
+                for (int hh = 0; hh < 2; ++hh) {  // lanes 32q + 16 hh .., rows r = 2 hh, 2 hh + 1
+                    uint32_t raw[32];
+                    tmem_ld16x256_x8(lane_base + ((uint32_t)(16 * hh) << 16) + kColS + sb * 128 + half * 64, raw);
                     tmem_wait_ld();
-                    if (ch == 1) {  // S of this warp read: the buffer may take the next tile
+                    if (hh == 1) {  // S of this warp read: the buffer may take the next tile
                         tc_fence_before();
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&s_empty[sb]);
                     }
                     uint32_t w[16];
-                    if (kt == t.qt) {  // the diagonal tile: causal mask, and the self term
-                        const int d0 = col0 - row;  // key minus query index of v[0]
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) v[c] = d0 + c <= 0 ? ex2(fmaf(v[c], a.scale_log2, -lrow)) : 0.f;
+                    for (int k = 0; k < 8; ++k) {
 #pragma unroll
-                        for (int c = 0; c < 32; c += 2) w[c >> 1] = pack_bf16(v[c], v[c + 1]);
-                        if (a.exclude_self) {
-#pragma unroll
-                            for (int c = 0; c < 32; ++c) v[c] = d0 + c == 0 ? 0.f : v[c];
+                        for (int rr = 0; rr < 2; ++rr) {
+                            const int r = 2 * hh + rr;
+                            float p0 = ex2(fmaf(__uint_as_float(raw[4 * k + 2 * rr]), a.scale_log2, -lr[r]));
+                            float p1 = ex2(fmaf(__uint_as_float(raw[4 * k + 2 * rr + 1]), a.scale_log2, -lr[r]));
+                            float c0 = p0, c1 = p1;
+                            if (diag) {  // causal mask, and the self term of the column sums
+                                const int dd = half * 64 + 8 * k + 2 * c4 - (q * 32 + g8 + 8 * r);
+                                p0 = dd <= 0 ? p0 : 0.f;
+                                p1 = dd + 1 <= 0 ? p1 : 0.f;
+                                c0 = a.exclude_self && dd == 0 ? 0.f : p0;
+                                c1 = a.exclude_self && dd + 1 == 0 ? 0.f : p1;
+                            }
+                            w[2 * k + rr] = pack_bf16(p0, p1);
+                            if (hh == 0 && rr == 0) {
+                                csum[2 * k] = c0;
+                                csum[2 * k + 1] = c1;
+                            } else {
+                                csum[2 * k] += c0;
+                                csum[2 * k + 1] += c1;
+                            }
                         }
-                    } else {  // every key precedes every query of the tile
-#pragma unroll
-                        for (int c = 0; c < 32; ++c) v[c] = ex2(fmaf(v[c], a.scale_log2, -lrow));
-#pragma unroll
-                        for (int c = 0; c < 32; c += 2) w[c >> 1] = pack_bf16(v[c], v[c + 1]);
                     }
-                    // P V of step - 2 has read this P buffer, and the reader warps have
-                    // added up this buffer's column sums of step - 2
-                    if (ch == 0 && step >= 2 &&
+                    // P V of step - 2 has read this P buffer
+                    if (hh == 0 && step >= 2 &&
                         !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
-                    tmem_st16(lane_base + kColP + sb * 64 + col0 / 2, w);
-                    const float sum = warp_reduce_scatter32(v);
-                    if (ch == 0 && step >= 2 &&
-                        !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
-                    csb[q * kT + col0 + lane] = sum;
+                    tmem_st16x128_x8(lane_base + ((uint32_t)(16 * hh) << 16) + kColP + sb * 64 + half * 32, w);
                 }
                 if (!ok) break;
+                // reduce-scatter over g8 (lane bits 2..4): lane (g8, c4) ends with columns
+                // 8 g8 + 2 c4 + 0..1 = 2 lane + 0..1 of the warp's 32 rows
+#pragma unroll
+                for (int lvl = 0; lvl < 3; ++lvl) {
+                    const int wdt = 8 >> lvl;            // values kept after this level
+                    const int bit = 16 >> lvl;           // lane bit exchanged
+                    const bool upper = (lane & bit) != 0;
+#pragma unroll
+                    for (int i = 0; i < wdt; ++i) {
+                        const float send = upper ? csum[i] : csum[i + wdt];
+                        const float keep = upper ? csum[i + wdt] : csum[i];
+                        csum[i] = keep + __shfl_xor_sync(0xffffffffu, send, bit);
+                    }
+                }
+                // the reducer warp is done with this buffer's sums of step - 2
+                if (step >= 2 && !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                *reinterpret_cast<float2*>(csb + q * kT + half * 64 + 2 * lane) = make_float2(csum[0], csum[1]);
                 asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 tc_fence_before();
                 __syncwarp();
