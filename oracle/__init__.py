@@ -60,6 +60,7 @@ class _Lib:
             "oracle_lm_head_entropy": [P, P, I, I64, I64, I64, I64, I64, P, I],
             "oracle_attn_lse": [P, P, I, I, I, I, D, P, I, P, I],
             "oracle_attn_output": [P, P, P, I, I, I, I, D, P, I, P, I],
+            "oracle_attn_output_rows": [P, P, P, I, I, I, I, D, P, I, I64, P, I],
             "oracle_attn_colsum": [P, P, I, I, I, I, D, P, I, P, I, I, P, I],
             "oracle_attn_colsum_rows": [P, P, I, I, I, I, D, P, I, P, I, I, I64, P, I],
             "oracle_importance": [P, P, I, I, I, P],
@@ -183,6 +184,21 @@ def attn_output(Q, K, V, cu_seqlens, scale, n_threads: int = 0) -> np.ndarray:
     _check(_load().oracle_attn_output(_ptr(Q), _ptr(K), _ptr(V), _dtype_code(Q), Hq, Hkv, d,
                                       float(scale), _ptr(cu), len(cu) - 1, _ptr(out), n_threads),
            "attn_output")
+    return out
+
+
+def attn_output_rows(Q, K, V, cu_seqlens, scale, row_from: int, n_threads: int = 0) -> np.ndarray:
+    """attn_output for the prompt-local query rows >= row_from; the other rows are 0."""
+    Q, K, V = np.ascontiguousarray(Q), np.ascontiguousarray(K), np.ascontiguousarray(V)
+    cu = _cu(cu_seqlens)
+    sumT, Hq, d = Q.shape
+    Hkv = K.shape[1]
+    assert K.shape == V.shape and K.dtype == Q.dtype == V.dtype
+    out = np.zeros((sumT, Hq, d), dtype=np.float64)
+    _check(_load().oracle_attn_output_rows(_ptr(Q), _ptr(K), _ptr(V), _dtype_code(Q), Hq, Hkv,
+                                           d, float(scale), _ptr(cu), len(cu) - 1,
+                                           int(row_from), _ptr(out), n_threads),
+           "attn_output_rows")
     return out
 
 

@@ -251,6 +251,7 @@ typedef struct {
     double scale;
     const int32_t* cu;
     double* O;
+    int64_t row_from; /* first prompt-local query row formed */
 } attn_out_ctx;
 
 /* One (prompt, query head) pair: for every query row i, the causal softmax row
@@ -274,7 +275,7 @@ static void attn_out_unit(void* vctx, int64_t unit, double* s) {
             v[t * d + x] = load_elem(c->V, c->dtype, row_kv * d + x);
         }
     }
-    for (int64_t i = 0; i < T; ++i) {
+    for (int64_t i = c->row_from; i < T; i++) {  /* output rows i >= row_from */
         double m = -INFINITY;
         for (int64_t j = 0; j <= i; ++j) {
             double dot = 0.0;
@@ -299,12 +300,20 @@ static void attn_out_unit(void* vctx, int64_t unit, double* s) {
 int oracle_attn_output(const void* Q, const void* K, const void* V, int dtype, int Hq, int Hkv,
                        int d, double scale, const int32_t* cu_seqlens, int B, double* O_out,
                        int n_threads) {
+    return oracle_attn_output_rows(Q, K, V, dtype, Hq, Hkv, d, scale, cu_seqlens, B, 0, O_out,
+                                   n_threads);
+}
+
+int oracle_attn_output_rows(const void* Q, const void* K, const void* V, int dtype, int Hq,
+                            int Hkv, int d, double scale, const int32_t* cu_seqlens, int B,
+                            int64_t row_from, double* O_out, int n_threads) {
+    if (row_from < 0) return -1;
     if (!valid_dtype(dtype) || Hq <= 0 || Hkv <= 0 || Hq % Hkv || d <= 0) return -1;
     if (!valid_cu(cu_seqlens, B)) return -1;
     const int64_t sumT = cu_seqlens[B];
     if (sumT == 0) return 0;
     if (!Q || !K || !V || !O_out) return -1;
-    attn_out_ctx c = {Q, K, V, dtype, Hq, Hkv, d, scale, cu_seqlens, O_out};
+    attn_out_ctx c = {Q, K, V, dtype, Hq, Hkv, d, scale, cu_seqlens, O_out, row_from};
     parallel_units(attn_out_unit, &c, (int64_t)B * Hq, (size_t)max_len(cu_seqlens, B), n_threads);
     return 0;
 }

@@ -69,6 +69,12 @@ int oracle_attn_output(const void* Q, const void* K, const void* V, int dtype, i
                        int d, double scale, const int32_t* cu_seqlens, int B, double* O_out,
                        int n_threads);
 
+/* The same output for the query rows i >= row_from (prompt-local index) only; the rows
+ * before are left as they are.  Used to check late rows of long prompts. */
+int oracle_attn_output_rows(const void* Q, const void* K, const void* V, int dtype, int Hq,
+                            int Hkv, int d, double scale, const int32_t* cu_seqlens, int B,
+                            int64_t row_from, double* O_out, int n_threads);
+
 /* Column sums of the causal softmax attention matrix of one layer, over a set of
  * query heads:  C_out[j] += sum_{h in heads} sum_{i >= j, i in prompt(j)} A^h_ij,
  * A^h_ij = softmax_j(scale * q_i^h . k_j^{h/rep}) over j <= i in the same prompt.

@@ -234,6 +234,33 @@ def pin_attn_output_bruteforce():
                what="attention output brute force")
 
 
+def pin_attn_output_rows_bruteforce():
+    """Output rows i >= row_from only (prompt-local index): those rows equal the brute-force
+    softmax rows times V (numpy / scipy), and the rows before stay 0."""
+    rng = _rng(63)
+    cu = np.asarray([0, 3, 3, 12, 13], np.int32)
+    Hq, Hkv, d, row_from = 4, 2, 16, 2
+    sumT = int(cu[-1])
+    Q = rng.standard_normal((sumT, Hq, d)).astype(np.float32)
+    K = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+    V = rng.standard_normal((sumT, Hkv, d)).astype(np.float32)
+    scale = 0.3
+    ref = np.zeros((sumT, Hq, d))
+    for b in range(len(cu) - 1):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        T = t1 - t0
+        if T == 0:
+            continue
+        for h in range(Hq):
+            g = h // (Hq // Hkv)
+            s = scale * Q[t0:t1, h].astype(np.float64) @ K[t0:t1, g].astype(np.float64).T
+            s[np.triu_indices(T, 1)] = -np.inf
+            full = special.softmax(s, axis=1) @ V[t0:t1, g].astype(np.float64)
+            ref[t0 + row_from:t1, h] = full[row_from:]
+    _close(oracle.attn_output_rows(Q, K, V, cu, scale, row_from), ref, rtol=1e-12, atol=1e-12,
+           what="attention output rows >= row_from")
+
+
 def pin_importance_bruteforce():
     """T <= 16: column sums of scipy softmax rows of the causal score matrix."""
     rng = _rng(3)

@@ -1,4 +1,4 @@
-"""Full-size importance and pooling on the three large workloads (GPU).
+"""Full-size importance, fused attention forward and pooling on the large workloads (GPU).
 
 The GPU runs the whole workload: every prompt, every selected layer and head, in
 per-layer calls that accumulate, as a caller streaming one layer's Q/K at a time
@@ -44,6 +44,50 @@ def test_importance_full_size(cuda_lib, w, R):
         Kp = _bits(K[t0:t1])
         oracle.attn_colsum_rows(Qp, Kp, sub, w.scale, T - R, out=C)
         del Q, K
+    S = ctx.attn_importance_finalize(len(w.layers), sumT).cpu().numpy()
+    ctx.sync_status()
+    assert np.all(np.isfinite(S)) and np.all(S >= 0)
+    sums = np.add.reduceat(S.astype(np.float64), cu[:-1])
+    assert np.max(np.abs(sums - 1.0)) < 1e-4, sums
+    ref = oracle.importance(C, sub, len(w.layers), w.Hq)[T - R:]
+    assert_importance(S[t1 - R:t1], ref)
+
+
+@pytest.mark.parametrize("w,R", [(W.C2, 8), (W.C3, 4), (W.C5, 4)],
+                         ids=lambda x: getattr(x, "name", str(x)))
+def test_forward_full_size(cuda_lib, w, R):
+    """The fused forward (estp_attn_forward_importance) over every selected layer of the
+    whole workload, row normalisers computed by the call, as the bench launches it. S is
+    finite, non-negative and sums to 1 over every prompt; the last R query rows of one
+    prompt (its O) and its last R keys (their importance) match the oracle."""
+    from test_gpu_attn_forward import O_TOL
+    import synth
+    cu = w.cu_seqlens()
+    sumT = int(cu[-1])
+    lens = np.diff(cu)
+    maxT = int(lens.max())
+    b = int(np.argmax(lens))
+    t0, t1 = int(cu[b]), int(cu[b + 1])
+    T = t1 - t0
+    ctx = cuda_lib.Context(0)
+    cu_d = sd.cu_seqlens(w)
+    C = np.zeros(T)
+    sub = np.asarray([0, T], dtype=np.int32)
+    for n, layer in enumerate(w.layers):
+        Q, K = sd.qk(w, layer)
+        V = sd.normal(w.key_v(layer), (sumT, w.Hkv, w.d), synth.BF16)
+        O = ctx.attn_forward_importance(Q, K, V, cu_d, maxT, accumulate=n > 0)
+        Qp = np.zeros((T, w.Hq, w.d), dtype=np.uint16)
+        Qp[T - R:] = _bits(Q[t1 - R:t1])
+        Kp, Vp = _bits(K[t0:t1]), _bits(V[t0:t1])
+        oracle.attn_colsum_rows(Qp, Kp, sub, w.scale, T - R, out=C)
+        if n == len(w.layers) - 1:
+            O_ref = oracle.attn_output_rows(Qp, Kp, Vp, sub, w.scale, T - R)[T - R:]
+            O_gpu = O[t1 - R:t1].float().cpu().numpy()
+            vmax = float(np.max(np.abs(synth.bf16_bits_to_f32(Vp))))
+            err = float(np.max(np.abs(O_gpu - O_ref)))
+            assert err <= O_TOL * vmax, f"O max abs err {err:.3e} (max|V| {vmax:.3e})"
+        del Q, K, V, O
     S = ctx.attn_importance_finalize(len(w.layers), sumT).cpu().numpy()
     ctx.sync_status()
     assert np.all(np.isfinite(S)) and np.all(S >= 0)

@@ -11,6 +11,8 @@ from oracle_pins import ALL_PINS
 # (what the mistake is, text in estp_oracle.c, replacement)
 MUTANTS = [
     ("entropy in bits", "H -= p * log(p);", "H -= p * log2(p);"),
+    ("output rows_from off by one", "for (int64_t i = c->row_from; i < T; i++) {",
+     "for (int64_t i = c->row_from + 1; i < T; i++) {"),
     ("entropy sign", "H -= p * log(p);", "H += p * log(p);"),
     ("entropy unnormalised", "double p = e[v] / s;", "double p = e[v];"),
     ("entropy ignores row stride", "int64_t off = r * c->ld;", "int64_t off = r * c->V;"),
