@@ -37,6 +37,8 @@
 // TMEM: S double-buffered (2 x 128 columns), O (128), P double-buffered (2 x 64 columns of
 // bf16 pairs): all 512.  Every mbarrier wait is bounded; on expiry the CTA records
 // ESTP_ERR_TIMEOUT and drains.
+#include <cstddef>
+
 #include "importance_tc.cuh"
 #include "tcgen05.cuh"
 
@@ -134,6 +136,11 @@ struct FwdItem {
     int pad;
 };
 constexpr int kSmemBytes = kItemOff + kSched * (int)sizeof(FwdItem) + 1024;
+// the decoded items are copied with 8-byte accesses at most: every slot and every int64
+// field must sit on an 8-byte boundary of the 1024-aligned shared-memory base
+static_assert(alignof(FwdItem) == 8 && sizeof(FwdItem) % 8 == 0, "FwdItem layout");
+static_assert(kItemOff % 8 == 0 && offsetof(FwdItem, t0) % 8 == 0 && offsetof(FwdItem, slot0) % 8 == 0,
+              "FwdItem alignment in shared memory");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
 __device__ __forceinline__ FwdItem fwd_item(const FwdArgs& a, int item) {
