@@ -1,6 +1,7 @@
 """Seeded random sweep of shapes against the oracle (GPU): combinations of ragged prompt
 lengths (empty prompts included), GQA ratios, head dims, head subsets, vocabulary and
-hidden sizes that the hand-picked cases of the other files do not cover one by one.
+hidden sizes that the hand-picked cases of the other files do not cover one by one,
+and the same for the fused prefill forward.
 Tolerances are the parity bar's (tests/gpu_util.py)."""
 import numpy as np
 import pytest
@@ -106,3 +107,20 @@ def test_sweep_lm_head(cuda_lib, seed):
     ctx.sync_status()
     bits = lambda t: t.view(torch.int16).cpu().numpy().view(np.uint16)
     assert_entropy(H.cpu().numpy(), oracle.lm_head_entropy(bits(h), bits(W)))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_sweep_attn_forward(cuda_lib, seed):
+    """Random lengths (empty prompts included), GQA ratio, self term, divisor, lse supplied
+    or computed, one or two layers through the fused forward (bf16, d 128)."""
+    from test_gpu_attn_forward import _run as _run_fwd
+    rng = np.random.default_rng(5000 + seed)
+    Hkv = int(rng.choice([1, 2, 4]))
+    Hq = Hkv * int(rng.choice([1, 3, 7]))
+    lens = _lens(rng, int(rng.integers(1, 7)), int(rng.choice([40, 300, 1500])))
+    w, cu = _wl(synth.BF16, lens, Hq, Hkv, 128, seed=seed + 70)
+    layers = [0] if rng.random() < 0.5 else [0, 1]
+    S, ref = _run_fwd(cuda_lib, w, cu, layers, exclude_self=bool(rng.random() < 0.3),
+                      supply_lse=bool(rng.random() < 0.5),
+                      divisor=str(rng.choice(["length", "causal", "none"])))
+    assert_importance(S, ref)
