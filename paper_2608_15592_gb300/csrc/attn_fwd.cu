@@ -169,9 +169,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* q_full = bars;           // [2]
     uint64_t* q_empty = bars + 2;      // [2]
     uint64_t* k_full = bars + 4;       // [2]
-    uint64_t* k_empty = bars + 6;      // [2]
+    // bars + 6, + 10: unused (a K or V^T slot is free when s_full / p_empty completes)
     uint64_t* v_full = bars + 8;       // [2]
-    uint64_t* v_empty = bars + 10;     // [2]
     uint64_t* s_full = bars + 12;      // [2]
     uint64_t* s_empty = bars + 14;     // [2]
     uint64_t* p_full = bars + 16;      // [2]
@@ -195,9 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&q_full[i], 1);
             mbar_init(&q_empty[i], 1);
             mbar_init(&k_full[i], 1);
-            mbar_init(&k_empty[i], 1);
             mbar_init(&v_full[i], 1);
-            mbar_init(&v_empty[i], 1);
             mbar_init(&s_full[i], 1);
             mbar_init(&s_empty[i], kGroupWarps);
             mbar_init(&p_full[i], kGroupWarps);
@@ -265,7 +262,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             auto load_v = [&](const VLoad& v) -> bool {
                 const int stage = (int)(v.step & 1);
                 const uint32_t u = v.step >> 1;
-                if (u >= 1 && !wait_bar(&v_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
+                // P V of step - 2 is complete (p_empty completes with it): its V^T slot is free
+                if (u >= 1 && !wait_bar(&p_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
                 mbar_expect_tx(&v_full[stage], kTileBytes);
                 for (int at = 0; at < 2; ++at)
                     tma_load_3d(sm + kVOff + stage * kTileBytes + at * kAtomBytes, &tm_vt,
@@ -298,7 +296,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int stage = (int)(step & 1);
                     const uint32_t u = step >> 1;
-                    if (u >= 1 && !wait_bar(&k_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                    // S of step - 2 is complete (s_full completes with it): its K slot is free
+                    if (u >= 1 && !wait_bar(&s_full[stage], (u - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
@@ -356,8 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_bf16<kIdesc>(tmem + kColS + stage * 128, sw128_desc(qa + off),
                                          sw128_desc(ka + off), kk > 0 ? 1u : 0u);
                     }
-                    mma_commit(&k_empty[stage]);
-                    mma_commit(&s_full[stage]);
+                    mma_commit(&s_full[stage]);  // also frees the K slot for the producer
                     if (kt == t.qt) mma_commit(&q_empty[fb]);  // the item's last use of Q
                 }
             }
@@ -393,8 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
                                sw128_desc(va + (kk >> 2) * kAtomBytes + (kk & 3) * 32),
                                (kt == 0 && kk == 0) ? 0u : 1u);
-                    mma_commit(&v_empty[pb]);
-                    mma_commit(&p_empty[pb]);
+                    mma_commit(&p_empty[pb]);  // also frees the V^T slot for the producer
                     if (kt == t.qt) mma_commit(&o_full[pb]);
                 }
             }
