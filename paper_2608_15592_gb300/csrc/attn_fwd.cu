@@ -461,7 +461,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 float* csb = cs + sb * 4 * kT;
                 const bool diag = kt == t.qt;
                 float csum[16];  // column sums of this thread's rows: [2k + e] for column 8k + 2c4 + e
-#pragma unroll 1
+                uint32_t w[2][16];  // packed P of both 16-lane halves, stored once all is computed
+#pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {  // lanes 32q + 16 hh .., rows r = 2 hh, 2 hh + 1
                     uint32_t raw[32];
                     tmem_ld16x256_x8(lane_base + ((uint32_t)(16 * hh) << 16) + kColS + sb * 128 + half * 64, raw);
@@ -471,7 +472,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&s_empty[sb]);
                     }
-                    uint32_t w[16];
 #pragma unroll
                     for (int k = 0; k < 8; ++k) {
 #pragma unroll
@@ -487,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 c0 = a.exclude_self && dd == 0 ? 0.f : p0;
                                 c1 = a.exclude_self && dd + 1 == 0 ? 0.f : p1;
                             }
-                            w[2 * k + rr] = pack_bf16(p0, p1);
+                            w[hh][2 * k + rr] = pack_bf16(p0, p1);
                             if (hh == 0 && rr == 0) {
                                 csum[2 * k] = c0;
                                 csum[2 * k + 1] = c1;
@@ -497,15 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     }
-                    // P V of step - 2 has read this P buffer
-                    if (hh == 0 && step >= 2 &&
-                        !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
-                        ok = false;
-                        break;
-                    }
-                    tmem_st16x128_x8(lane_base + ((uint32_t)(16 * hh) << 16) + kColP + sb * 64 + half * 32, w);
                 }
-                if (!ok) break;
                 // reduce-scatter over g8 (lane bits 2..4): lane (g8, c4) ends with columns
                 // 8 g8 + 2 c4 + 0..1 = 2 lane + 0..1 of the warp's 32 rows
 #pragma unroll
@@ -526,6 +518,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 *reinterpret_cast<float2*>(csb + q * kT + half * 64 + 2 * lane) = make_float2(csum[0], csum[1]);
+                // P V of step - 2 has read this P buffer
+                if (step >= 2 && !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                tmem_st16x128_x8(lane_base + kColP + sb * 64 + half * 32, w[0]);
+                tmem_st16x128_x8(lane_base + (16u << 16) + kColP + sb * 64 + half * 32, w[1]);
                 asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 tc_fence_before();
                 __syncwarp();
