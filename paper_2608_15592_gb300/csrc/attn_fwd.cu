@@ -20,9 +20,10 @@
 // 16-byte aligned, and the padding is zero.
 //
 // attn_fwd_kernel: one persistent CTA per SM, 320 threads.
-//   warp 0      TMA producer: claims items, stages Q (2 buffers), K and V^T of each key
-//               tile (a ring of 2 each: a K tile is free once S is computed, a V^T tile
-//               once P V is)
+//   warp 0      TMA producer: claims items, stages Q (1 buffer: the next item's Q loads
+//               once the item's last S is done), K (a ring of 3: a load takes ~1500 cycles,
+//               a slot frees when its S is done) and V^T (a ring of 2, a slot frees when
+//               its P V is done)
 //   warp 1      issues S = Q K^T (as soon as a K tile and an S buffer are free)
 //   warp 2      issues O += P V (as soon as the epilogue has written P): two issuing
 //               threads, because one thread that issues 16 MMAs, makes 4 barrier checks
@@ -55,12 +56,15 @@ constexpr int kRedWarp = kEpiWarp0 + kEpiWarps;  // the column-sum reducer
 constexpr int kThreads = 32 * (kRedWarp + 1);
 constexpr int kSched = 4;
 // dynamic shared memory (offsets from a 1024-aligned base)
-constexpr int kQOff = 0;                          // [2] Q tiles
-constexpr int kKOff = 2 * kTileBytes;             // [2 stages] K tiles
-constexpr int kVOff = 4 * kTileBytes;             // [2 stages] V^T tiles
-constexpr int kCsOff = 6 * kTileBytes;            // [2][4 quarters][128] column sums
+constexpr int kQBufs = 1;                         // Q tiles (the next item's Q loads
+                                                  // once the last S of the item is done)
+constexpr int kKStages = 3;                       // K ring: a K load takes ~1500 cycles
+constexpr int kQOff = 0;
+constexpr int kKOff = kQBufs * kTileBytes;
+constexpr int kVOff = kKOff + kKStages * kTileBytes;  // [2 stages] V^T tiles
+constexpr int kCsOff = kVOff + 2 * kTileBytes;        // [2][4 quarters][128] column sums
 constexpr int kBarOff = kCsOff + 2 * 4 * kT * 4;
-constexpr int kNumBars = 20 + 5 + 4 + 2 * kSched;
+constexpr int kNumBars = 2 * kQBufs + 2 * kKStages + 2 + 8 + 3 + 2 + 4 + 2 * kSched;
 constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem address, abort flag
 constexpr int kItemOff = kMiscOff + 16;           // [kSched] decoded items of the sched ring
 // TMEM columns
@@ -166,23 +170,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                                              ~uintptr_t(1023));
     float* cs = reinterpret_cast<float*>(sm + kCsOff);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kBarOff);
-    uint64_t* q_full = bars;           // [2]
-    uint64_t* q_empty = bars + 2;      // [2]
-    uint64_t* k_full = bars + 4;       // [2]
-    // bars + 6, + 10: unused (a K or V^T slot is free when s_full / p_empty completes)
-    uint64_t* v_full = bars + 8;       // [2]
-    uint64_t* s_full = bars + 12;      // [2]
-    uint64_t* s_empty = bars + 14;     // [2]
-    uint64_t* p_full = bars + 16;      // [2]
-    uint64_t* p_empty = bars + 18;     // [2]
+    uint64_t* q_full = bars;                         // [kQBufs]
+    uint64_t* q_empty = q_full + kQBufs;             // [kQBufs]
+    uint64_t* k_full = q_empty + kQBufs;             // [kKStages]
+    uint64_t* k_empty = k_full + kKStages;           // [kKStages]
+    uint64_t* v_full = k_empty + kKStages;           // [2] (a V^T slot is free when p_empty completes)
+    uint64_t* s_full = v_full + 2;                   // [2]
+    uint64_t* s_empty = s_full + 2;                  // [2]
+    uint64_t* p_full = s_empty + 2;                  // [2]
+    uint64_t* p_empty = p_full + 2;                  // [2]
     // [2] O complete, for the group that takes the parity of the item's last step: each
     // group waits on every phase of its own barrier
-    uint64_t* o_full = bars + 20;
-    uint64_t* o_empty = bars + 22;
-    uint64_t* drain = bars + 23;       // [2] each issuer's MMAs done
-    uint64_t* cs_full = bars + 25;     // [2] column sums of every quarter written
-    uint64_t* cs_empty = bars + 27;    // [2] column sums added up by the reducer warp
-    uint64_t* sched_full = bars + 29;  // [kSched]
+    uint64_t* o_full = p_empty + 2;
+    uint64_t* o_empty = o_full + 2;
+    uint64_t* drain = o_empty + 1;     // [2] each issuer's MMAs done
+    uint64_t* cs_full = drain + 2;     // [2] column sums of every quarter written
+    uint64_t* cs_empty = cs_full + 2;  // [2] column sums added up by the reducer warp
+    uint64_t* sched_full = cs_empty + 2;  // [kSched]
     uint64_t* sched_empty = sched_full + kSched;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kMiscOff + 4);
@@ -190,10 +194,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kQBufs; ++i) {
             mbar_init(&q_full[i], 1);
             mbar_init(&q_empty[i], 1);
+        }
+        for (int i = 0; i < kKStages; ++i) {
             mbar_init(&k_full[i], 1);
+            mbar_init(&k_empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(&v_full[i], 1);
             mbar_init(&s_full[i], 1);
             mbar_init(&s_empty[i], kGroupWarps);
@@ -285,8 +294,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(&sched_full[slot]);
                 if (item < 0) break;
                 const int g = t.h / (a.Hq / a.Hkv);
-                const int fb = it & 1;
-                if (it >= 2 && !wait_bar(&q_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
+                const int fb = it % kQBufs;
+                if (it >= kQBufs && !wait_bar(&q_empty[fb], ((it / kQBufs) - 1) & 1, abort_flag, a.status)) break;
                 mbar_expect_tx(&q_full[fb], kTileBytes);
                 for (int at = 0; at < 2; ++at)
                     tma_load_3d(sm + kQOff + fb * kTileBytes + at * kAtomBytes, &tm_q, at * 64, t.h,
@@ -294,10 +303,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ++n_items;
                 const int pstart = t.pos0;
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
-                    const int stage = (int)(step & 1);
-                    const uint32_t u = step >> 1;
-                    // S of step - 2 is complete (s_full completes with it): its K slot is free
-                    if (u >= 1 && !wait_bar(&s_full[stage], (u - 1) & 1, abort_flag, a.status)) {
+                    const int stage = (int)(step % kKStages);
+                    const uint32_t u = step / kKStages;
+                    if (u >= 1 && !wait_bar(&k_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
                         ok = false;
                         break;
                     }
@@ -320,12 +328,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (ok && have_v && load_v(vp)) ++v_issued;
             // every copy in flight lands before the CTA exits
-            for (uint32_t i = 0; i < 2 && i < step; ++i)
-                drain_wait(&k_full[(step - 1 - i) & 1], ((step - 1 - i) >> 1) & 1, a.status);
+            for (uint32_t i = 0; i < (uint32_t)kKStages && i < step; ++i)
+                drain_wait(&k_full[(step - 1 - i) % kKStages], ((step - 1 - i) / kKStages) & 1, a.status);
             for (uint32_t i = 0; i < 2 && i < v_issued; ++i)
                 drain_wait(&v_full[(v_issued - 1 - i) & 1], ((v_issued - 1 - i) >> 1) & 1, a.status);
-            for (int fb = 0; fb < 2 && fb < n_items; ++fb)
-                drain_wait(&q_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
+            for (int i = 0; i < kQBufs && i < n_items; ++i) {  // the last load of each Q buffer
+                const int last = n_items - 1 - i;
+                drain_wait(&q_full[last % kQBufs], (uint32_t)((last / kQBufs) & 1), a.status);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ S issuer
@@ -335,27 +345,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int it = 0; ok; ++it) {
                 const FwdItem t = consume_item(it, false);
                 if (!t.valid) break;
-                const int fb = it & 1;
-                if (!wait_bar(&q_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
+                const int fb = it % kQBufs;
+                if (!wait_bar(&q_full[fb], (it / kQBufs) & 1, abort_flag, a.status)) break;
                 const uint32_t qa = smem_u32(sm + kQOff + fb * kTileBytes);
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
-                    const int stage = (int)(step & 1);
+                    const int kst = (int)(step % kKStages);
+                    const int stage = (int)(step & 1);  // S buffer
                     const uint32_t u = step >> 1;
-                    if (!wait_bar(&k_full[stage], u & 1, abort_flag, a.status) ||
+                    if (!wait_bar(&k_full[kst], (step / kKStages) & 1, abort_flag, a.status) ||
                         (u >= 1 && !wait_bar(&s_empty[stage], (u - 1) & 1, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     issued = true;
-                    const uint32_t ka = smem_u32(sm + kKOff + stage * kTileBytes);
+                    const uint32_t ka = smem_u32(sm + kKOff + kst * kTileBytes);
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
                         const uint32_t off = (uint32_t)((kk >> 2) * kAtomBytes + (kk & 3) * 32);
                         mma_bf16<kIdesc>(tmem + kColS + stage * 128, sw128_desc(qa + off),
                                          sw128_desc(ka + off), kk > 0 ? 1u : 0u);
                     }
-                    mma_commit(&s_full[stage]);  // also frees the K slot for the producer
+                    mma_commit(&k_empty[kst]);
+                    mma_commit(&s_full[stage]);
                     if (kt == t.qt) mma_commit(&q_empty[fb]);  // the item's last use of Q
                 }
             }
