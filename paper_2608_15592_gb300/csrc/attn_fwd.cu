@@ -235,8 +235,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // the plans (and the lse values) are complete past this point
+    // the plans, V^T (and the lse values) are complete past this point
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int total = a.info->ok && a.info2->ok ? a.info->total : 0;
 
     // the k-th item of this CTA, decoded by the producer (valid = 0: no more items)
@@ -589,6 +590,8 @@ __global__ void __launch_bounds__(256) vt_transpose_kernel(const __nv_bfloat16* 
                                                            int Hq, int Hkv, int64_t L,
                                                            __nv_bfloat16* __restrict__ Vt) {
     __shared__ __align__(16) uint16_t tile[kTrPos][kD + 8];  // [position][d], rows padded by 16 bytes
+    asm volatile("griddepcontrol.wait;" ::: "memory");             // the plan is complete
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");  // the forward's prologue may start
     const int g = blockIdx.y;
     const int64_t p0 = (int64_t)blockIdx.x * kTrPos;
     const int32_t n_tiles = base[B] / Hq;
@@ -626,6 +629,7 @@ __global__ void __launch_bounds__(32 * kRedHeadLanes)
                           const PlanInfo* info, const PlanInfo* info2, int B, int Hq, int64_t sumT,
                           int accumulate, float* acc) {
     __shared__ float red[kRedHeadLanes][32];
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // the forward's partial slots are complete
     const int jj = threadIdx.x & 31, hl = threadIdx.x >> 5;
     const int64_t j = (int64_t)blockIdx.x * 32 + jj;
     float v = 0.f;
@@ -719,8 +723,25 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     // plans: items (prompt, query tile, head), and the partial slots (tile pairs x heads)
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, ctx->status);
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 2, base2, info2, ctx->status);
-    vt_transpose_kernel<<<dim3((unsigned)(L / kTrPos), (unsigned)Hkv), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(V), cu, base, B, Hq, Hkv, L, Vt);
+    // the transpose, the forward and the reduce are programmatic dependents of the launch
+    // before them: each starts its prologue early and waits on the device for its inputs
+    cudaLaunchAttribute pdl[1];
+    pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    auto config = [&](dim3 grid, dim3 block, size_t smem) {
+        cudaLaunchConfig_t c = {};
+        c.gridDim = grid;
+        c.blockDim = block;
+        c.dynamicSmemBytes = smem;
+        c.stream = st;
+        c.attrs = pdl;
+        c.numAttrs = 1;
+        return c;
+    };
+    cudaLaunchConfig_t ctr = config(dim3((unsigned)(L / kTrPos), (unsigned)Hkv), dim3(256), 0);
+    cudaError_t e = cudaLaunchKernelEx(&ctr, vt_transpose_kernel, static_cast<const __nv_bfloat16*>(V),
+                                       cu, (const int32_t*)base, B, Hq, Hkv, L, Vt);
+    if (e != cudaSuccess) return cuda_fail(e, "V transpose launch");
     CUtensorMap mq, mk, mvt;
     // Q, K: (d, head, token), one head's 64 x 128 atom per box; V^T: (position, d, head)
     if ((s = make_map3(&mq, Q, kD, Hq, sumT, (uint64_t)kD * 2, (uint64_t)Hq * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
@@ -732,13 +753,15 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     a.scale_log2 = scale * kLog2e;
     a.exclude_self = exclude_self ? 1 : 0;
     a.lse = lse; a.O = static_cast<__nv_bfloat16*>(O); a.part = part; a.status = ctx->status;
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward smem attribute");
-    attn_fwd_kernel<<<(unsigned)ctx->num_sms, kThreads, kSmemBytes, st>>>(mq, mk, mvt, a);
-    e = cudaGetLastError();
+    cudaLaunchConfig_t cf = config(dim3((unsigned)ctx->num_sms), dim3(kThreads), kSmemBytes);
+    e = cudaLaunchKernelEx(&cf, attn_fwd_kernel, mq, mk, mvt, a);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward launch");
-    imp_fwd_reduce_kernel<<<(unsigned)((sumT + 31) / 32), 32 * kRedHeadLanes, 0, st>>>(
-        part, cu, base2, info, info2, B, Hq, sumT, accumulate ? 1 : 0, acc);
+    cudaLaunchConfig_t cr = config(dim3((unsigned)((sumT + 31) / 32)), dim3(32 * kRedHeadLanes), 0);
+    e = cudaLaunchKernelEx(&cr, imp_fwd_reduce_kernel, (const float*)part, cu, (const int32_t*)base2,
+                           (const PlanInfo*)info, (const PlanInfo*)info2, B, Hq, sumT, accumulate ? 1 : 0, acc);
+    if (e != cudaSuccess) return cuda_fail(e, "attention forward reduce launch");
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "attention forward reduce launch");
 }
