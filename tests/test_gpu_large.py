@@ -53,7 +53,7 @@ def test_importance_full_size(cuda_lib, w, R):
     assert_importance(S[t1 - R:t1], ref)
 
 
-@pytest.mark.parametrize("w,R", [(W.C2, 8), (W.C3, 4), (W.C5, 4)],
+@pytest.mark.parametrize("w,R", [(W.C2, 8), (W.C3, 4), (W.C4, 8), (W.C5, 4)],
                          ids=lambda x: getattr(x, "name", str(x)))
 def test_forward_full_size(cuda_lib, w, R):
     """The fused forward (estp_attn_forward_importance) over every selected layer of the
