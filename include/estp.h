@@ -192,9 +192,8 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
  *   out : bf16 [sumT, Hq, 128] (device, 16-byte aligned), written for every token.
  *   dtype must be ESTP_BF16 and head_dim 128 (else ESTP_ERR_UNSUPPORTED).
  * The probabilities enter O = A V rounded to bf16 (as a flash-attention forward does);
- * the column sums use them unrounded.  The workspace holds V^T (2 * Hkv * 128 bytes per
- * position, prompts padded to 128) and one fp32 row of 128 column sums per (head, query
- * tile, key tile <= query tile). */
+ * the column sums use them unrounded.  The workspace holds one fp32 row of 128 column sums
+ * per (head, query tile, key tile <= query tile). */
 estp_status estp_attn_forward_importance(estp_ctx* ctx, const void* Q, const void* K,
                                          const void* V, estp_dtype dtype, const float* lse,
                                          int32_t Hq, int32_t Hkv, int32_t head_dim,

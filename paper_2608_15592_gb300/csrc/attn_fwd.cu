@@ -8,21 +8,21 @@
 // rescale, on the tensor cores:
 //   S   = Q K^T       tcgen05.mma, M = N = 128, K = 16 x 8 steps over d = 128, into TMEM
 //   P   = 2^(S scale log2e - lse log2e)   epilogue, written back to TMEM as bf16
-//   O  += P V         tcgen05.mma with A = P from TMEM, B = the key tile of V^T
+//   O  += P V         tcgen05.mma with A = P from TMEM, B = the key tile of V
 // and the column sums of P over the tile's 128 query rows (a warp reduce-scatter, then the
 // four TMEM lane quarters in order) go to a partial buffer, one slot per (prompt, head,
 // query tile, key tile).  imp_fwd_reduce_kernel adds a key's slots in a fixed order into
 // the accumulator: no floating-point atomics, repeated calls give identical bits.
 //
-// V enters the second MMA as its transpose V^T [Hkv][d][positions], written by
-// vt_transpose_kernel, so that it is K-major (keys contiguous) like every other operand;
-// each prompt starts at a multiple of 128 positions, which keeps every TMA coordinate
-// 16-byte aligned, and the padding is zero.
+// V enters the second MMA as it is stored, [sumT, Hkv, 128]: a 128-key tile lands in shared
+// memory as rows of keys with d contiguous, which is B in the MN-major form (N = d
+// contiguous, 128-byte swizzle; the two 64-wide d blocks 16 KB apart, the 8-key groups
+// 1 KB apart).  Keys past the prompt meet P = 0.
 //
 // attn_fwd_kernel: one persistent CTA per SM, 320 threads.
 //   warp 0      TMA producer: claims items, stages Q (1 buffer: the next item's Q loads
 //               once the item's last S is done), K (a ring of 3: a load takes ~1500 cycles,
-//               a slot frees when its S is done) and V^T (a ring of 2, a slot frees when
+//               a slot frees when its S is done) and V (a ring of 2, a slot frees when
 //               its P V is done)
 //   warp 1      issues S = Q K^T (as soon as a K tile and an S buffer are free)
 //   warp 2      issues O += P V (as soon as the epilogue has written P): two issuing
@@ -61,7 +61,7 @@ constexpr int kQBufs = 1;                         // Q tiles (the next item's Q 
 constexpr int kKStages = 3;                       // K ring: a K load takes ~1500 cycles
 constexpr int kQOff = 0;
 constexpr int kKOff = kQBufs * kTileBytes;
-constexpr int kVOff = kKOff + kKStages * kTileBytes;  // [2 stages] V^T tiles
+constexpr int kVOff = kKOff + kKStages * kTileBytes;  // [2 stages] V tiles
 constexpr int kCsOff = kVOff + 2 * kTileBytes;        // [2][4 quarters][128] column sums
 constexpr int kBarOff = kCsOff + 2 * 4 * kT * 4;
 constexpr int kNumBars = 2 * kQBufs + 2 * kKStages + 2 + 8 + 3 + 2 + 4 + 2 * kSched;
@@ -70,6 +70,15 @@ constexpr int kItemOff = kMiscOff + 16;           // [kSched] decoded items of t
 // TMEM columns
 constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdesc = idesc_bf16(kT, kT);   // M = N = 128 for both products
+constexpr uint32_t kIdescPV = kIdesc | (1u << 16);  // P V: B (the V tile) MN-major
+
+// Shared-memory descriptor of an MN-major B tile with 128-byte swizzle: 64 d values per
+// 128-byte row of one key, 8-key groups 1 KB apart (stride byte offset), the second
+// 64-wide d block 16 KB on (leading byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t addr) {
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)(16384 >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
 
 struct FwdArgs {
     const int32_t* cu;
@@ -87,13 +96,13 @@ struct FwdArgs {
     int* status;
 };
 
-// A operand from TMEM: D (TMEM) = A (TMEM) B^T (+ D when acc != 0).
+// O += P V: A from TMEM, B an MN-major shared-memory tile (+ D when acc != 0).
 __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t acc) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "r"(a_tmem), "l"(b), "r"(kIdesc), "r"(acc));
+        "r"(a_tmem), "l"(b), "r"(kIdescPV), "r"(acc));
 }
 
 // tcgen05.ld .16x256b.x8: 16 lanes from the lane of taddr, 64 columns.  Thread t gets, for
@@ -136,8 +145,6 @@ struct FwdItem {
     int h, qt, T;
     int64_t t0;
     int64_t slot0;          // partial slot of (this head, query tile, key tile 0)
-    int pos0;               // V^T position of the prompt's first key
-    int pad;
 };
 constexpr int kSmemBytes = kItemOff + kSched * (int)sizeof(FwdItem) + 1024;
 // the decoded items are copied with 8-byte accesses at most: every slot and every int64
@@ -157,14 +164,12 @@ __device__ __forceinline__ FwdItem fwd_item(const FwdArgs& a, int item) {
     t.T = li.T;
     const int nt = (li.T + kT - 1) / kT;
     t.slot0 = a.base2[li.b] + (int64_t)li.hslot * tri(nt) + tri(li.qt);
-    t.pos0 = (a.base[li.b] / a.Hq) * kT;
-    t.pad = 0;
     return t;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_vt, const FwdArgs a) {
+                    const __grid_constant__ CUtensorMap tm_v, const FwdArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -260,8 +265,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_q)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_vt)) : "memory");
-            // V^T of step s is issued after K of step s + 1: it is needed one MMA pair
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v)) : "memory");
+            // V of step s is issued after K of step s + 1: it is needed one MMA pair
             // later, and its ring slot frees later
             struct VLoad {
                 int pos, g;
@@ -276,8 +281,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (u >= 1 && !wait_bar(&p_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
                 mbar_expect_tx(&v_full[stage], kTileBytes);
                 for (int at = 0; at < 2; ++at)
-                    tma_load_3d(sm + kVOff + stage * kTileBytes + at * kAtomBytes, &tm_vt,
-                                v.pos + at * 64, 0, v.g, &v_full[stage]);
+                    tma_load_3d(sm + kVOff + stage * kTileBytes + at * kAtomBytes, &tm_v,
+                                at * 64, v.g, v.pos, &v_full[stage]);
                 return true;
             };
             uint32_t step = 0, v_issued = 0;
@@ -302,7 +307,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_3d(sm + kQOff + fb * kTileBytes + at * kAtomBytes, &tm_q, at * 64, t.h,
                                 (int)(t.t0 + t.qt * kT), &q_full[fb]);
                 ++n_items;
-                const int pstart = t.pos0;
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int stage = (int)(step % kKStages);
                     const uint32_t u = step / kKStages;
@@ -321,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         ++v_issued;
                     }
-                    vp = VLoad{pstart + kt * kT, g, step};
+                    vp = VLoad{(int)(t.t0 + kt * kT), g, step};
                     have_v = true;
                 }
                 if (!ok) break;
@@ -402,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)
                         mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                               sw128_desc(va + (kk >> 2) * kAtomBytes + (kk & 3) * 32),
+                               sw128_mn_desc(va + kk * 16 * 128),  // keys 16 kk ..
                                (kt == 0 && kk == 0) ? 0u : 1u);
                     mma_commit(&p_empty[pb]);  // also frees the V^T slot for the producer
                     if (kt == t.qt) mma_commit(&o_full[pb]);
@@ -580,46 +584,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// V [sumT, Hkv, 128] -> V^T [Hkv][128][L], prompt b's tokens at positions pstart_b ..,
-// pstart_b = 128 * (tiles of the prompts before b); the padding after each prompt is zero.
-// A block moves 64 positions (inside one prompt's 128-aligned span) x 128 d of one KV head
-// through shared memory, with 16-byte loads and stores on both sides.
-constexpr int kTrPos = 64;
-__global__ void __launch_bounds__(256) vt_transpose_kernel(const __nv_bfloat16* __restrict__ V,
-                                                           const int32_t* cu, const int32_t* base, int B,
-                                                           int Hq, int Hkv, int64_t L,
-                                                           __nv_bfloat16* __restrict__ Vt) {
-    __shared__ __align__(16) uint16_t tile[kTrPos][kD + 8];  // [position][d], rows padded by 16 bytes
-    asm volatile("griddepcontrol.wait;" ::: "memory");             // the plan is complete
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");  // the forward's prologue may start
-    const int g = blockIdx.y;
-    const int64_t p0 = (int64_t)blockIdx.x * kTrPos;
-    const int32_t n_tiles = base[B] / Hq;
-    int64_t src0 = 0, n_valid = 0;  // first source token of the block, tokens that exist
-    if (p0 < (int64_t)n_tiles * kT) {
-        const int b = upper_slot(base, B, (int)(p0 / kT) * Hq);
-        const int64_t tl0 = p0 - (int64_t)(base[b] / Hq) * kT;
-        src0 = cu[b] + tl0;
-        n_valid = min((int64_t)kTrPos, (int64_t)(cu[b + 1] - cu[b]) - tl0);
-    }
-    for (int c = threadIdx.x; c < kTrPos * (kD / 8); c += blockDim.x) {
-        const int r = c / (kD / 8), q = c % (kD / 8);  // position r, d values 8q .. 8q + 7
-        uint4 val = make_uint4(0, 0, 0, 0);
-        if (r < n_valid)
-            val = *reinterpret_cast<const uint4*>(V + ((src0 + r) * Hkv + g) * (int64_t)kD + q * 8);
-        *reinterpret_cast<uint4*>(&tile[r][q * 8]) = val;
-    }
-    __syncthreads();
-    for (int c = threadIdx.x; c < kD * (kTrPos / 8); c += blockDim.x) {
-        const int dd = c / (kTrPos / 8), q = c % (kTrPos / 8);  // d row dd, positions 8q .. 8q + 7
-        uint32_t w[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            w[k] = (uint32_t)tile[q * 8 + 2 * k][dd] | ((uint32_t)tile[q * 8 + 2 * k + 1][dd] << 16);
-        *reinterpret_cast<uint4*>(Vt + ((int64_t)g * kD + dd) * L + p0 + q * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-    }
-}
-
 // C_j (+)= sum over heads h and query tiles qt >= kt(j) of the partial slots of key j.  A block
 // takes 32 keys; its warp w sums heads w, w + 8, .. (each over qt in order), and the 8 warp
 // sums are added in order: a fixed order, whatever the launch.
@@ -687,12 +651,11 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
                                 const int32_t* cu, int B, int64_t sumT, int max_seqlen,
                                 bool exclude_self, bool accumulate, float* acc, void* O,
                                 cudaStream_t st) {
-    // workspace: V^T | partial slots | lse (when not given) | plans | row-normaliser plan
+    // workspace: partial slots | lse (when not given) | plans | row-normaliser plan
     const int64_t max_nt = (max_seqlen + kT - 1) / kT;
     const int64_t tiles_bound = (sumT + kT - 1) / kT + B;          // sum of nt_b
-    const int64_t L = tiles_bound * kT;                             // V^T positions
     const int64_t slots_bound = (int64_t)Hq * tiles_bound * (max_nt + 1) / 2 + Hq;
-    const size_t off_part = align_up(sizeof(__nv_bfloat16) * (size_t)Hkv * kD * (size_t)L, 256);
+    const size_t off_part = 0;
     const size_t off_lse = off_part + align_up(sizeof(float) * (size_t)slots_bound * kT, 256);
     const size_t off_plan = off_lse + (lse_in ? 0 : align_up(sizeof(float) * (size_t)Hq * sumT, 256));
     const size_t off_base2 = off_plan + align_up(sizeof(int32_t) * (size_t)(B + 1), 256);
@@ -704,7 +667,6 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
                                         sizeof(PlanInfo) + 256);
     if (s != ESTP_OK) return s;
     char* ws = static_cast<char*>(ctx->ws);
-    __nv_bfloat16* Vt = reinterpret_cast<__nv_bfloat16*>(ws);
     float* part = reinterpret_cast<float*>(ws + off_part);
     int32_t* base = reinterpret_cast<int32_t*>(ws + off_plan);
     int32_t* base2 = reinterpret_cast<int32_t*>(ws + off_base2);
@@ -723,8 +685,8 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     // plans: items (prompt, query tile, head), and the partial slots (tile pairs x heads)
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, ctx->status);
     attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 2, base2, info2, ctx->status);
-    // the transpose, the forward and the reduce are programmatic dependents of the launch
-    // before them: each starts its prologue early and waits on the device for its inputs
+    // the forward and the reduce are programmatic dependents of the launch before them:
+    // each starts its prologue early and waits on the device for its inputs
     cudaLaunchAttribute pdl[1];
     pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     pdl[0].val.programmaticStreamSerializationAllowed = 1;
@@ -738,15 +700,12 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
         c.numAttrs = 1;
         return c;
     };
-    cudaLaunchConfig_t ctr = config(dim3((unsigned)(L / kTrPos), (unsigned)Hkv), dim3(256), 0);
-    cudaError_t e = cudaLaunchKernelEx(&ctr, vt_transpose_kernel, static_cast<const __nv_bfloat16*>(V),
-                                       cu, (const int32_t*)base, B, Hq, Hkv, L, Vt);
-    if (e != cudaSuccess) return cuda_fail(e, "V transpose launch");
-    CUtensorMap mq, mk, mvt;
-    // Q, K: (d, head, token), one head's 64 x 128 atom per box; V^T: (position, d, head)
+    cudaError_t e;
+    CUtensorMap mq, mk, mv;
+    // Q, K, V: (d, head, token), one head's 64 d x 128 tokens per box
     if ((s = make_map3(&mq, Q, kD, Hq, sumT, (uint64_t)kD * 2, (uint64_t)Hq * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
     if ((s = make_map3(&mk, K, kD, Hkv, sumT, (uint64_t)kD * 2, (uint64_t)Hkv * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
-    if ((s = make_map3(&mvt, Vt, L, kD, Hkv, (uint64_t)L * 2, (uint64_t)L * kD * 2, 64, kD, 1)) != ESTP_OK) return s;
+    if ((s = make_map3(&mv, V, kD, Hkv, sumT, (uint64_t)kD * 2, (uint64_t)Hkv * kD * 2, 64, 1, kT)) != ESTP_OK) return s;
     FwdArgs a{};
     a.cu = cu; a.base = base; a.base2 = base2; a.info = info; a.info2 = info2;
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.sumT = sumT;
@@ -756,7 +715,7 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward smem attribute");
     cudaLaunchConfig_t cf = config(dim3((unsigned)ctx->num_sms), dim3(kThreads), kSmemBytes);
-    e = cudaLaunchKernelEx(&cf, attn_fwd_kernel, mq, mk, mvt, a);
+    e = cudaLaunchKernelEx(&cf, attn_fwd_kernel, mq, mk, mv, a);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward launch");
     cudaLaunchConfig_t cr = config(dim3((unsigned)((sumT + 31) / 32)), dim3(32 * kRedHeadLanes), 0);
     e = cudaLaunchKernelEx(&cr, imp_fwd_reduce_kernel, (const float*)part, cu, (const int32_t*)base2,
