@@ -74,6 +74,7 @@ CASES = [
     ([0, 0, 200], 2, 2),
     ([257, 64, 63, 513], 28, 4),
     ([1100], 4, 2),
+    ([300, 50, 129], 64, 1),   # GQA ratio 64: one KV head for every query head
 ]
 
 
@@ -147,3 +148,31 @@ def test_forward_rejects_unsupported(cuda_lib):
     Q32 = torch.zeros(8, 2, 128, dtype=torch.float32, device="cuda")
     with pytest.raises(cuda_lib.EstpError):
         ctx.attn_forward_importance(Q32, Q32, Q32, cu, 8)    # fp32
+
+
+def test_forward_rejects_bad_arguments(cuda_lib):
+    """Host-side validation, before any launch: misaligned V or output, a NULL V, and
+    accumulate = 1 without an open accumulation."""
+    ctx = cuda_lib.Context(0)
+    cu = torch.tensor([0, 8], dtype=torch.int32, device="cuda")
+    Q = torch.zeros(8, 2, 128, dtype=torch.bfloat16, device="cuda")
+    K = torch.zeros(8, 1, 128, dtype=torch.bfloat16, device="cuda")
+    flat = torch.zeros(8 * 128 + 8, dtype=torch.bfloat16, device="cuda")
+    V_mis = flat[1:1 + 8 * 128].view(8, 1, 128)            # 2 bytes off a 16-byte boundary
+    with pytest.raises(cuda_lib.EstpError):
+        ctx.attn_forward_importance(Q, K, V_mis, cu, 8)
+    out_flat = torch.zeros(8 * 2 * 128 + 8, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(cuda_lib.EstpError):
+        ctx.attn_forward_importance(Q, K, K, cu, 8, out=out_flat[1:1 + 8 * 2 * 128].view(8, 2, 128))
+    import ctypes
+    lib = cuda_lib.lib
+    rc = lib.estp_attn_forward_importance(ctx._h, Q.data_ptr(), K.data_ptr(), None, 1, None, 2, 1, 128,
+                                          0.1, cu.data_ptr(), 1, 8, 8, 0, 0, Q.data_ptr(), None)
+    assert rc != 0
+    ctx2 = cuda_lib.Context(0)
+    with pytest.raises(cuda_lib.EstpError):
+        ctx2.attn_forward_importance(Q, K, K, cu, 8, accumulate=True)
+    # a valid call still works on the same context afterwards
+    O = ctx.attn_forward_importance(Q, K, K, cu, 8)
+    ctx.sync_status()
+    assert O.shape == (8, 2, 128)
