@@ -475,7 +475,7 @@ def time_attn_forward(st, peak_tflops, kern_ms, iters: int = 20, warmup_s: float
     out = {"ms_per_layer": ms_fused, "ms_per_layer_with_lse": ms_internal,
            "layers": n_layers, "flops_per_layer": alg, "bound": "tensor", "achieved": tf,
            "unit": "TFLOP/s", "peak": peak_tflops, "frac": tf / peak_tflops,
-           "launches_per_layer": 4, "unfused_importance_ms_per_layer":
+           "launches_per_layer": 3, "unfused_importance_ms_per_layer":
            kern_ms["lse"] + kern_ms["importance"]}
     try:
         import torch.nn.functional as F

@@ -683,8 +683,8 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
         lse = l;
     }
     // plans: items (prompt, query tile, head), and the partial slots (tile pairs x heads)
-    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, ctx->status);
-    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 2, base2, info2, ctx->status);
+    attn_plan2_kernel<<<2, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kT, 1, Hq, 1, base, info, 2, base2,
+                                          info2, ctx->status);
     // the forward and the reduce are programmatic dependents of the launch before them:
     // each starts its prologue early and waits on the device for its inputs
     cudaLaunchAttribute pdl[1];

@@ -14,13 +14,10 @@
 
 namespace estp {
 
-__global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int B, int64_t sumT,
-                                                         int max_seqlen, int tile, int qc,
-                                                         int mult, int kind, int32_t* base,
-                                                         PlanInfo* info, int* status) {
-    // the tensor-core kernel that consumes the plan may launch now and run its prologue;
-    // it waits for this grid before its first read of the plan
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+// One plan, computed by all 1024 threads of the calling block.
+static __device__ void plan_body(const int32_t* cu, int B, int64_t sumT, int max_seqlen, int tile,
+                                 int qc, int mult, int kind, int32_t* base, PlanInfo* info,
+                                 int* status) {
     // thread t owns prompts [t*per, (t+1)*per); one read of cu, warp-shuffle scans
     __shared__ int64_t warp_sum[32];
     __shared__ int bad;
@@ -71,6 +68,27 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
         info->next = 0;
     }
     if (tid == 0 && !ok) report(status, ESTP_ERR_INVALID_ARG);
+}
+
+__global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int B, int64_t sumT,
+                                                         int max_seqlen, int tile, int qc,
+                                                         int mult, int kind, int32_t* base,
+                                                         PlanInfo* info, int* status) {
+    // the tensor-core kernel that consumes the plan may launch now and run its prologue;
+    // it waits for this grid before its first read of the plan
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    plan_body(cu, B, sumT, max_seqlen, tile, qc, mult, kind, base, info, status);
+}
+
+__global__ void __launch_bounds__(1024) attn_plan2_kernel(const int32_t* cu, int B, int64_t sumT,
+                                                          int max_seqlen, int tile, int qc,
+                                                          int mult, int kind0, int32_t* base0,
+                                                          PlanInfo* info0, int kind1,
+                                                          int32_t* base1, PlanInfo* info1,
+                                                          int* status) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (blockIdx.x == 0) plan_body(cu, B, sumT, max_seqlen, tile, qc, mult, kind0, base0, info0, status);
+    else plan_body(cu, B, sumT, max_seqlen, tile, qc, mult, kind1, base1, info1, status);
 }
 
 namespace {

@@ -41,6 +41,15 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const int32_t* cu, int 
                                                          int mult, int kind, int32_t* base,
                                                          PlanInfo* info, int* status);
 
+// Two plans of the same prompts in one launch of 2 blocks: block 0 writes (kind0, base0,
+// info0), block 1 (kind1, base1, info1).
+__global__ void __launch_bounds__(1024) attn_plan2_kernel(const int32_t* cu, int B, int64_t sumT,
+                                                          int max_seqlen, int tile, int qc,
+                                                          int mult, int kind0, int32_t* base0,
+                                                          PlanInfo* info0, int kind1,
+                                                          int32_t* base1, PlanInfo* info1,
+                                                          int* status);
+
 struct ImpItem {
     int b, g, kt, qt0, qt1;
     int64_t t0;
