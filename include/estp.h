@@ -102,8 +102,9 @@ estp_status estp_token_entropy(estp_ctx* ctx, const void* logits, estp_dtype dty
  *   - All calls share the array, and it keeps the last call's contents: calls that
  *     overlap on the GPU (different streams, or concurrent host threads) race on it.
  *     Order them on one stream.
- *   - A GPU whose launch would need more than 4096 partial pairs (more than ~170 SMs
- *     at the kernel's occupancy) gets ESTP_ERR_WORKSPACE and nothing is enqueued.
+ *   - The launch uses at most 4096 pieces (one per warp).  A GPU with more resident
+ *     warps than that (more than ~170 SMs at the kernel's occupancy) runs with fewer,
+ *     longer pieces: the result is the same, only the split differs.
  * Errors are reported as for estp_token_entropy; there is no device status word. */
 estp_status estp_token_entropy_noalloc(const void* logits, estp_dtype dtype, int64_t n_rows,
                                        int64_t V, int64_t ld, float* entropy_out,

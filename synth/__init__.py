@@ -54,18 +54,35 @@ def uniform24(key: int, n) -> np.ndarray:
     return (w >> np.uint64(40)).astype(np.float64) * (1.0 / (1 << 24))
 
 
+def _splitmix64_inplace(key: int, n: np.ndarray) -> np.ndarray:
+    """splitmix64(key, n) computed in the buffer n (uint64, overwritten)."""
+    with np.errstate(over="ignore"):
+        z = n
+        z += np.uint64(1)
+        z *= GAMMA
+        z += np.uint64(key)
+        z ^= z >> np.uint64(30)
+        z *= _M1
+        z ^= z >> np.uint64(27)
+        z *= _M2
+        z ^= z >> np.uint64(31)
+    return z
+
+
 def normal(key: int, idx) -> np.ndarray:
-    """Irwin-Hall normal draws for element indices ``idx`` (exact binary64)."""
+    """Irwin-Hall normal draws for element indices ``idx`` (exact binary64): the sum of
+    the twelve 16-bit pieces of words 3 idx, 3 idx + 1 and 3 idx + 2."""
     idx = np.asarray(idx, dtype=np.uint64).reshape(-1)
     out = np.empty(idx.shape, dtype=np.float64)
-    for s in range(0, idx.size, _CHUNK):
-        n = idx[s:s + _CHUNK]
-        acc = np.zeros(n.shape, dtype=np.int64)
+    chunk = _CHUNK >> 2
+    for s in range(0, idx.size, chunk):
+        n3 = idx[s:s + chunk] * np.uint64(3)
+        acc = np.zeros(n3.shape, dtype=np.int64)
         for k in range(3):
-            w = splitmix64(key, n * np.uint64(3) + np.uint64(k))
-            for c in range(4):
-                acc += ((w >> np.uint64(16 * c)) & np.uint64(0xFFFF)).astype(np.int64)
-        out[s:s + _CHUNK] = (acc + 6).astype(np.float64) * (1.0 / 65536.0) - 6.0
+            w = _splitmix64_inplace(key, n3 + np.uint64(k))
+            # the four 16-bit pieces of each word (their order does not matter for the sum)
+            acc += w.view(np.uint16).reshape(-1, 4).sum(axis=1, dtype=np.int64)
+        out[s:s + chunk] = (acc + 6).astype(np.float64) * (1.0 / 65536.0) - 6.0
     return out
 
 

@@ -141,17 +141,31 @@ def host_hidden(w: Workload, rows) -> np.ndarray:
     return round_to(normal(w.key(S_HIDDEN), idx), w.dtype).reshape(rows.size, w.D)
 
 
-def host_qk(w: Workload, layer: int, rows=None):
-    """Q [n, Hq, d] and K [n, Hkv, d] of one layer for global token rows (all by default),
-    with the sink rows of K scaled."""
-    cu = w.cu_seqlens()
+def _rows(w: Workload, rows):
     if rows is None:
-        rows = np.arange(int(cu[-1]))
-    rows = np.asarray(rows, dtype=np.int64).reshape(-1)
+        rows = np.arange(int(w.cu_seqlens()[-1]))
+    return np.asarray(rows, dtype=np.int64).reshape(-1)
+
+
+def host_q(w: Workload, layer: int, rows=None) -> np.ndarray:
+    """Q [n, Hq, d] of one layer for global token rows (all by default)."""
+    rows = _rows(w, rows)
     qi = (rows[:, None] * (w.Hq * w.d) + np.arange(w.Hq * w.d)[None, :]).reshape(-1)
+    return round_to(normal(w.key_q(layer), qi), w.dtype).reshape(rows.size, w.Hq, w.d)
+
+
+def host_k(w: Workload, layer: int, rows=None) -> np.ndarray:
+    """K [n, Hkv, d] of one layer for global token rows (all by default), with the sink
+    rows scaled."""
+    rows = _rows(w, rows)
     ki = (rows[:, None] * (w.Hkv * w.d) + np.arange(w.Hkv * w.d)[None, :]).reshape(-1)
-    Q = round_to(normal(w.key_q(layer), qi), w.dtype).reshape(rows.size, w.Hq, w.d)
     K64 = normal(w.key_k(layer), ki).reshape(rows.size, w.Hkv, w.d)
     sink = np.isin(rows, w.sink_rows())
     K64[sink] *= w.sink_scale
-    return Q, round_to(K64, w.dtype).reshape(rows.size, w.Hkv, w.d)
+    return round_to(K64, w.dtype).reshape(rows.size, w.Hkv, w.d)
+
+
+def host_qk(w: Workload, layer: int, rows=None):
+    """Q [n, Hq, d] and K [n, Hkv, d] of one layer for global token rows (all by default),
+    with the sink rows of K scaled."""
+    return host_q(w, layer, rows), host_k(w, layer, rows)

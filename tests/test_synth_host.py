@@ -68,3 +68,21 @@ def test_sinks_scaled():
     assert np.array_equal(Kf[sink], 8 * Pf[sink])
     rest = [i for i in range(12) if i not in sink]
     assert np.array_equal(Kf[rest], Pf[rest])
+
+
+def test_normal_matches_scalar_definition():
+    # Irwin-Hall normal of index i: the twelve 16-bit pieces of SplitMix64 words 3i, 3i+1
+    # and 3i+2, summed, plus 6, times 2**-16, minus 6 -- evaluated with Python integers.
+    def word(key, n):
+        z = (key + (n + 1) * 0x9E3779B97F4A7C15) & (2**64 - 1)
+        z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & (2**64 - 1)
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & (2**64 - 1)
+        return z ^ (z >> 31)
+
+    key = synth.stream_key(5, 77)
+    idx = [0, 1, 2, 1000, 123456789, (1 << 40) + 3]
+    want = []
+    for i in idx:
+        acc = sum((word(key, 3 * i + k) >> (16 * c)) & 0xFFFF for k in range(3) for c in range(4))
+        want.append((acc + 6) / 65536.0 - 6.0)
+    assert list(synth.normal(key, idx)) == want
