@@ -5,8 +5,9 @@ owns all of HBM for its KV cache, or code running where cudaMalloc is not allowe
 estp_token_entropy_noalloc serves them with the partials kept in a static device
 array.  This test calls it through the C ABI and checks it against
 estp_token_entropy on two calls in a row (the second call reuses the static array
-with whatever the first call left in it).  The file sorts last so that a run that
-stops at the first failure has already run every other test.
+with whatever the first call left in it), and against the fp64 oracle on the same
+rows.  The file sorts last so that a run that stops at the first failure has already
+run every other test.
 """
 import ctypes
 
@@ -14,7 +15,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import ENTROPY_ATOL
+import oracle
+from gpu_util import ENTROPY_ATOL, assert_entropy
 from synth import device as sd
 from synth import workloads as W
 
@@ -43,9 +45,15 @@ def test_noalloc_matches_entropy_twice(cuda_lib):
             torch.cuda.synchronize()
             outs.append(out.cpu().numpy())
         r = ref.cpu().numpy()
+        if x.dtype == torch.bfloat16:
+            xh = x.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        else:
+            xh = x.cpu().numpy()
+        exact = oracle.token_entropy(xh, V=V)
         for o in outs:
             assert np.all(np.isfinite(o))
             assert np.max(np.abs(o - r)) <= ENTROPY_ATOL
+            assert_entropy(o, exact)
     ctx.close()
 
 
