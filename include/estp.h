@@ -72,6 +72,18 @@ const char* estp_last_error(const estp_ctx* ctx);
  * (ESTP_OK, ESTP_ERR_INVALID_ARG for bad varlen metadata, ESTP_ERR_TIMEOUT). */
 estp_status estp_sync_status(estp_ctx* ctx, estp_stream_t stream);
 
+/* Testing aid for the failure path; the paper has no counterpart.  Sets, for this
+ * context's later calls, the limit in SM clock cycles of the abortable waits of the
+ * tensor-core attention kernels (the row normalisers and column sums of
+ * estp_attn_lse / estp_attn_importance on bf16 inputs).  cycles <= 0 restores the
+ * default, about 2 s.  A limit far below a tile copy's latency makes those waits
+ * expire: each CTA then records ESTP_ERR_TIMEOUT in the status word, skips the rest of
+ * its work, and waits (with the full default limit) for the copies and MMAs it has
+ * already issued before it frees its tensor memory and exits, so the context stays
+ * usable.  The outputs of a call that timed out are undefined; estp_sync_status
+ * returns ESTP_ERR_TIMEOUT.  Host-side only: nothing is enqueued. */
+estp_status estp_set_wait_limit(estp_ctx* ctx, int64_t cycles);
+
 /* ------------------------------------------------------------------ (a)
  * Token entropy, Eq. 2-1 (Sec. 3.2):
  *   entropy_out[r] = -sum_{v<V} p_rv ln p_rv,  p_r = softmax(logits[r, 0:V]),

@@ -37,7 +37,8 @@ EXPORTS = ("estp_create", "estp_destroy", "estp_last_error", "estp_sync_status",
            "estp_token_entropy", "estp_attn_lse", "estp_attn_importance",
            "estp_attn_importance_finalize", "estp_pool", "estp_token_entropy_noalloc",
            "estp_head_loss", "estp_misalignment", "estp_lm_head_entropy",
-           "estp_mlp_head_predict", "estp_mlp_head_loss", "estp_attn_forward_importance")
+           "estp_mlp_head_predict", "estp_mlp_head_loss", "estp_attn_forward_importance",
+           "estp_set_wait_limit")
 
 
 class EstpError(RuntimeError):
@@ -80,6 +81,7 @@ def _load():
         "estp_destroy": ([P], None),
         "estp_last_error": ([P], ctypes.c_char_p),
         "estp_sync_status": ([P, P], ctypes.c_int),
+        "estp_set_wait_limit": ([P, I64], ctypes.c_int),
         "estp_token_entropy": ([P, P, ctypes.c_int, I64, I64, I64, P, I32, P, P], ctypes.c_int),
         "estp_attn_lse": ([P, P, P, ctypes.c_int, I32, I32, I32, F, P, I32, I64, I32, P, P],
                           ctypes.c_int),
@@ -177,6 +179,11 @@ class Context:
     def sync_status(self, stream=None):
         """estp_sync_status: synchronise the stream; raise on a device-side error."""
         _check(lib.estp_sync_status(self._h, _stream(stream)))
+
+    def set_wait_limit(self, cycles: int = 0):
+        """estp_set_wait_limit: limit (SM cycles) of the attention kernels' abortable
+        waits for later calls; 0 restores the default.  A testing aid."""
+        _check(lib.estp_set_wait_limit(self._h, int(cycles)))
 
     # ------------------------------------------------------------------ (a)
     def lm_head_entropy(self, hidden, W, out=None, stream=None):

@@ -132,7 +132,14 @@ void estp_destroy(estp_ctx* ctx) {
 
 const char* estp_last_error(const estp_ctx*) { return g_msg; }
 
+estp_status estp_set_wait_limit(estp_ctx* ctx, int64_t cycles) {
+    if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
+    ctx->wait_cycles = cycles > 0 ? (long long)cycles : kWaitCycles;
+    return ESTP_OK;
+}
+
 estp_status estp_sync_status(estp_ctx* ctx, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_sync_status");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     estp_status st = set_device(ctx);
     if (st != ESTP_OK) return st;
@@ -157,6 +164,7 @@ estp_status estp_token_entropy(estp_ctx* ctx, const void* logits, estp_dtype dty
                                int64_t n_rows, int64_t V, int64_t ld,
                                const int32_t* cu_seqlens, int32_t B, float* entropy_out,
                                estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_token_entropy");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (dtype != ESTP_F32 && dtype != ESTP_BF16) return fail(ESTP_ERR_INVALID_ARG, "dtype");
     if (n_rows < 0 || V < 1 || ld < V)
@@ -197,6 +205,7 @@ estp_status estp_attn_lse(estp_ctx* ctx, const void* Q, const void* K, estp_dtyp
                           int32_t Hq, int32_t Hkv, int32_t head_dim, float softmax_scale,
                           const int32_t* cu_seqlens, int32_t B, int64_t sumT,
                           int32_t max_seqlen, float* lse_out, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_attn_lse");
     estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
                                 B, sumT, max_seqlen);
     if (st != ESTP_OK) return st;
@@ -266,6 +275,7 @@ estp_status estp_attn_importance(estp_ctx* ctx, const void* Q, const void* K,
                                  int32_t n_heads, const int32_t* cu_seqlens, int32_t B,
                                  int64_t sumT, int32_t max_seqlen, int accumulate,
                                  uint32_t flags, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_attn_importance");
     estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
                                 B, sumT, max_seqlen);
     if (st != ESTP_OK) return st;
@@ -287,6 +297,7 @@ estp_status estp_attn_forward_importance(estp_ctx* ctx, const void* Q, const voi
                                          int32_t B, int64_t sumT, int32_t max_seqlen,
                                          int accumulate, uint32_t flags, void* out,
                                          estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_attn_forward_importance");
     estp_status st = check_attn(ctx, Q, K, dtype, Hq, Hkv, head_dim, softmax_scale, cu_seqlens,
                                 B, sumT, max_seqlen);
     if (st != ESTP_OK) return st;
@@ -305,6 +316,7 @@ estp_status estp_attn_forward_importance(estp_ctx* ctx, const void* Q, const voi
 
 estp_status estp_attn_importance_finalize(estp_ctx* ctx, int32_t n_layers,
                                           float* importance_out, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_attn_importance_finalize");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (!ctx->imp_open) return fail(ESTP_ERR_INVALID_ARG, "no open importance accumulation");
     if (n_layers < 1) return fail(ESTP_ERR_INVALID_ARG, "n_layers must be >= 1");
@@ -322,6 +334,7 @@ estp_status estp_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int64
                       const int32_t* cu_seqlens, int32_t B, int64_t sumT,
                       estp_mix_params mix, const estp_head* head, float* pooled_out,
                       float* pred_len_out, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_pool");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (dtype != ESTP_F32 && dtype != ESTP_BF16) return fail(ESTP_ERR_INVALID_ARG, "dtype");
     if (D < 1 || ldh < D || B < 0 || sumT < 0 || sumT > INT32_MAX)
@@ -348,6 +361,7 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
                            const estp_head* head, const float* targets, float lambda3,
                            float* loss_out, float* grad_W, float* grad_bias,
                            float* grad_pooled, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_head_loss");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (B < 1 || D < 1) return fail(ESTP_ERR_INVALID_ARG, "need B >= 1 and D >= 1");
     if (!head || !head->W || !head->centers || head->K < 1 || head->K > 1024)
@@ -363,6 +377,7 @@ estp_status estp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, int64_
 estp_status estp_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ldh, const void* W,
                                  int64_t ldw, estp_dtype dtype, int64_t n_rows, int64_t D,
                                  int64_t V, float* entropy_out, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_lm_head_entropy");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (dtype != ESTP_BF16) return fail(ESTP_ERR_UNSUPPORTED, "lm-head entropy: bf16 only");
     if (n_rows < 0 || D < 64 || D % 64 || V < 1)
@@ -394,6 +409,7 @@ static estp_status check_mlp(estp_ctx* ctx, const float* pooled, int32_t B, int6
 estp_status estp_mlp_head_predict(estp_ctx* ctx, const float* pooled, int32_t B, int64_t D,
                                   const estp_mlp_head* head, float* pred_out, float* probs_out,
                                   estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_mlp_head_predict");
     estp_status st = check_mlp(ctx, pooled, B, D, head);
     if (st != ESTP_OK) return st;
     if (!pred_out) return fail(ESTP_ERR_INVALID_ARG, "NULL tensor pointer");
@@ -407,6 +423,7 @@ estp_status estp_mlp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, in
                                const estp_mlp_head* head, const float* targets, float lambda3,
                                float* loss_out, const estp_mlp_grads* grads,
                                estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_mlp_head_loss");
     estp_status st = check_mlp(ctx, pooled, B, D, head);
     if (st != ESTP_OK) return st;
     if (!std::isfinite(lambda3)) return fail(ESTP_ERR_INVALID_ARG, "lambda3 must be finite");
@@ -421,6 +438,7 @@ estp_status estp_mlp_head_loss(estp_ctx* ctx, const float* pooled, int32_t B, in
 estp_status estp_misalignment(estp_ctx* ctx, const float* entropy, const float* importance,
                               const int32_t* cu_seqlens, int32_t B, int64_t sumT, int32_t pct,
                               int32_t* counts_out, estp_stream_t stream) {
+    ESTP_NVTX_RANGE("estp_misalignment");
     if (!ctx) return fail(ESTP_ERR_INVALID_ARG, "ctx is NULL");
     if (B < 0 || sumT < 0 || sumT > INT32_MAX)
         return fail(ESTP_ERR_INVALID_ARG, "need B >= 0 and 0 <= sumT < 2^31");

@@ -369,6 +369,7 @@ extern "C" estp_status estp_token_entropy_noalloc(const void* logits, estp_dtype
                                                   int64_t n_rows, int64_t V, int64_t ld,
                                                   float* entropy_out, estp_stream_t stream) {
     using namespace estp;
+    ESTP_NVTX_RANGE("estp_token_entropy_noalloc");
     if (dtype != ESTP_F32 && dtype != ESTP_BF16) return fail(ESTP_ERR_INVALID_ARG, "dtype");
     if (n_rows < 0 || V < 1 || ld < V)
         return fail(ESTP_ERR_INVALID_ARG, "need n_rows >= 0, V >= 1, ld >= V");

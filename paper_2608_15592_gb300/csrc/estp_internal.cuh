@@ -5,7 +5,12 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "estp.h"
+
+// Bounded device waits: about 2 s of SM clock.
+constexpr long long kWaitCycles = 4000000000ll;
 
 struct estp_ctx {
     int device = 0;
@@ -24,9 +29,21 @@ struct estp_ctx {
     uint32_t imp_flags = 0;     // flags of the opening call (divisor variant, self term)
     uint32_t* pool_done = nullptr;      // per-prompt arrival counters of the pooling kernel
     int32_t pool_done_cap = 0;
+    // limit of the attention kernels' abortable waits (estp_set_wait_limit)
+    long long wait_cycles = kWaitCycles;
 };
 
 namespace estp {
+
+// An NVTX range named after the entry point for the length of the host call (a no-op
+// unless a profiler is attached), so that a timeline groups each call's launches.
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
+#define ESTP_NVTX_RANGE(name) ::estp::NvtxRange estp_nvtx_range_(name)
 
 // ---------------------------------------------------------------- host helpers
 estp_status fail(estp_status st, const char* fmt, ...);

@@ -33,8 +33,11 @@
 //   stays in the thread that owns key j; a tile skips query tiles before its own key
 //   tile.
 //
-// Every mbarrier wait is bounded (about 2 s of SM clock); on expiry the CTA records
-// ESTP_ERR_TIMEOUT in the status word and drains without further waits.
+// Every mbarrier wait is bounded (about 2 s of SM clock; a test may lower the limit of
+// the abortable waits through estp_set_wait_limit); on expiry the CTA records
+// ESTP_ERR_TIMEOUT in the status word, skips every further abortable wait, and drains:
+// the producer waits (full limit) for its last copies into each ring slot, fixed-tile
+// buffer and lse slot, the issuers for all their MMAs, before the TMEM is freed.
 #include "importance_tc.cuh"
 #include "tcgen05.cuh"
 
@@ -94,6 +97,7 @@ struct TcArgs {
     float* part;        // column-sum mode output [c][G][sumT]
     float* lse_out;     // LSE mode output [Hq, sumT]
     int* status;
+    long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
     ImpHeads hs;
 };
 
@@ -265,8 +269,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = k % kSched;
         const uint32_t par = (uint32_t)((k / kSched) & 1);
         bool got;
-        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
-        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
+        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status, a.wait_cycles);
+        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status, a.wait_cycles);
         if (!got) return -1;
         const int item = sched_item[slot];
         if (warp_uniform) __syncwarp();
@@ -282,20 +286,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (MODE == kModeImp)
                 asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_lse)) : "memory");
             uint32_t step = 0;
+            // lse copies issued: one per step, issued before the step's ring wait, so an
+            // abort at that wait leaves one more lse copy than ring copies in flight
+            uint32_t lse_issued = 0;
             int n_items = 0;
             int item = blockIdx.x;
             for (int it = 0;; ++it) {
                 if (item >= total) item = -1;
                 const int slot = it % kSched;
                 if (it >= kSched &&
-                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
+                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status, a.wait_cycles))
                     break;
                 sched_item[slot] = item;
                 mbar_arrive(&sched_full[slot]);  // release: the item index is visible to waiters
                 if (item < 0) break;
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
-                if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status)) break;
+                if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 mbar_expect_tx(&fix_full[fb], 2 * C::kTileBytes);
 #pragma unroll
                 for (int tau = 0; tau < 2; ++tau)
@@ -314,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (MODE == kModeImp) {  // the tile's lse values, from a 16-byte boundary
                         const int ls = (int)(step % kLseSlots);
                         const uint32_t lu = step / kLseSlots;
-                        if (lu >= 1 && !wait_bar(&lse_empty[ls], (lu - 1) & 1, abort_flag, a.status)) {
+                        if (lu >= 1 && !wait_bar(&lse_empty[ls], (lu - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                             ok = false;
                             break;
                         }
@@ -322,8 +329,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mbar_expect_tx(&lse_full[ls], kLseBox * 4);
                         tma_load_1d(lse_ring + ls * (kLseSlotBytes / 4), &tm_lse, (int)(x & ~int64_t(3)),
                                     &lse_full[ls]);
+                        ++lse_issued;
                     }
-                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                    if (u >= 1 && !wait_bar(&ring_empty[stage], (u - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                         ok = false;
                         break;
                     }
@@ -343,8 +351,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 drain_wait(&ring_full[(step - 1 - st) % C::kStages], ((step - 1 - st) / C::kStages) & 1,
                            a.status);
             if (MODE == kModeImp)
-                for (uint32_t ls = 0; ls < (uint32_t)kLseSlots && ls < step; ++ls)
-                    drain_wait(&lse_full[ls], ((step - 1 - ls) / kLseSlots) & 1, a.status);
+                for (uint32_t k = 0; k < (uint32_t)kLseSlots && k < lse_issued; ++k) {
+                    const uint32_t s2 = lse_issued - 1 - k;  // the last copy into each slot
+                    drain_wait(&lse_full[s2 % kLseSlots], (s2 / kLseSlots) & 1, a.status);
+                }
             for (int fb = 0; fb < 2 && fb < n_items; ++fb)
                 drain_wait(&fix_full[fb], (uint32_t)(((n_items - 1 - fb) / 2) & 1), a.status);
         }
@@ -359,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (item < 0) break;
                 const TcItem t = make_item<MODE>(a, item);
                 const int fb = it & 1;
-                if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status)) break;
+                if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 const uint32_t fix_addr = smem_u32(fix + (fb * 2 + tau) * C::kTileBytes);
                 bool ok = true;
                 for (int s = 0; s < t.n_steps; ++s, ++step) {
@@ -368,11 +378,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int ab = (int)(step % kAccBufs);
                     const uint32_t ua = step / kAccBufs;
                     const uint32_t str_addr = smem_u32(ring + stage * C::kTileBytes);
-                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status)) {
+                    if (!wait_bar(&ring_full[stage], u & 1, abort_flag, a.status, a.wait_cycles)) {
                         ok = false;
                         break;
                     }
-                    if (ua >= 1 && !wait_bar(&acc_empty[tau * kAccBufs + ab], (ua - 1) & 1, abort_flag, a.status)) {
+                    if (ua >= 1 && !wait_bar(&acc_empty[tau * kAccBufs + ab], (ua - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                         ok = false;
                         break;
                     }
@@ -423,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int row0 = si.row0, head = si.head, qt = si.qt;
                 if (MODE == kModeImp) {  // -log2e * lse of the step's 128 query columns
                     const int ls = (int)(step % kLseSlots);
-                    if (!warp_wait(&lse_full[ls], (step / kLseSlots) & 1, abort_flag, a.status))
+                    if (!warp_wait(&lse_full[ls], (step / kLseSlots) & 1, abort_flag, a.status, a.wait_cycles))
                         return false;
                     const int64_t x = (int64_t)head * a.sumT + t.t0 + row0;
                     const float* lr = lse_ring + ls * (kLseSlotBytes / 4) + (int)(x & 3);
@@ -441,7 +451,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 const int ab = (int)(step % kAccBufs);
                 const int abar = tau * kAccBufs + ab;  // accumulator barrier
-                if (!warp_wait(&acc_full[abar], (step / kAccBufs) & 1, abort_flag, a.status))
+                if (!warp_wait(&acc_full[abar], (step / kAccBufs) & 1, abort_flag, a.status, a.wait_cycles))
                     return false;
                 tc_fence_after();
                 // column-sum mode: this warp's key tile against the streamed query tile
@@ -540,14 +550,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint64_t* xf = &xfull[(pb * 2 + tau) * 4 + q];
             uint64_t* xe = &xempty[(pb * 2 + tau) * 4 + q];
             if (sub == 1) {
-                if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status);
+                if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status, a.wait_cycles);
                 if (!ok) break;
                 mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
                                                      : make_float2(m, ssum);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(xf);
             } else {
-                ok = warp_wait(xf, use & 1, abort_flag, a.status);
+                ok = warp_wait(xf, use & 1, abort_flag, a.status, a.wait_cycles);
                 if (!ok) break;
                 const float2 o = mb[q * 32 + lane];
                 __syncwarp();
@@ -653,6 +663,7 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
     a.scale_log2 = scale * kLog2e;
     a.lse_out = lse;
     a.status = ctx->status;
+    a.wait_cycles = ctx->wait_cycles;
     a.hs = hs;
     CUtensorMap mq, mk;
     if ((s = make_map(&mq, Q, Hq, d, sumT)) != ESTP_OK) return s;
@@ -678,6 +689,7 @@ estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const flo
     a.lse = lse;
     a.part = part;
     a.status = ctx->status;
+    a.wait_cycles = ctx->wait_cycles;
     a.hs = hs;
     // the lse coordinate of a TMA copy is a 32-bit element index
     if ((int64_t)Hq * sumT + kLseBox >= ((int64_t)1 << 31))

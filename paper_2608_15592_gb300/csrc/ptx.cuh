@@ -6,8 +6,6 @@
 
 namespace estp {
 
-constexpr long long kWaitCycles = 4000000000ll;  // bounded waits: about 2 s of SM clock
-
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
@@ -43,15 +41,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait: false (and the CTA's abort flag set) when the barrier does not
-// complete in time or another role of the CTA has already aborted.
+// complete within `limit` SM cycles or another role of the CTA has already aborted.
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status) {
+                                         int* status, long long limit = kWaitCycles) {
     if (mbar_try_wait(bar, parity)) return true;  // fast path: no flag read
     if (*abort_flag) return false;
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity)) {
         if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitCycles) {
+        if (clock64() - t0 > limit) {
             *abort_flag = 1;
             report(status, ESTP_ERR_TIMEOUT);
             return false;
@@ -60,7 +58,9 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
     return true;
 }
 
-// Bounded wait that ignores the abort flag (used to drain outstanding async work).
+// Bounded wait that ignores the abort flag (used to drain outstanding async work); its
+// limit is always the full kWaitCycles, so that every copy and MMA a CTA issued has
+// completed before it frees its tensor memory and exits.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* status) {
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity)) {
@@ -73,21 +73,12 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
 
 // Warp-uniform bounded wait: lane 0 polls, every lane gets the same answer.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
+                                          int* status, long long limit = kWaitCycles) {
     bool r = false;
-    if ((threadIdx.x & 31) == 0) r = wait_bar(bar, parity, abort_flag, status);
+    if ((threadIdx.x & 31) == 0) r = wait_bar(bar, parity, abort_flag, status, limit);
     r = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0;
     __syncwarp();
     return r;
-}
-
-// Untiled bulk copy global -> shared (both 16-byte aligned, size a multiple of 16).
-__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            smem_u32(dst)),
-        "l"(src), "r"(bytes), "r"(smem_u32(bar))
-        : "memory");
 }
 
 // max of three floats in one instruction (sm_100+)
@@ -97,102 +88,5 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     return d;
 }
 
-__device__ __forceinline__ void named_bar(int id, int n) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
-}
-
 }  // namespace estp
 
-// ------------------------------------------------------------- cluster helpers
-namespace estp {
-
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-__device__ __forceinline__ uint32_t cluster_id_x() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
-    return r;
-}
-
-__device__ __forceinline__ uint32_t nclusters_x() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
-    return r;
-}
-
-// Address in CTA `rank` of the cluster of the shared variable at `addr` in this CTA.
-__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-    return r;
-}
-
-__device__ __forceinline__ void st_cluster_s32(uint32_t addr, int v) {
-    asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-
-// Arrival (release at cluster scope) on an mbarrier of any CTA of the cluster.
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t addr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(addr)
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// wait_bar / drain_wait for barriers that other CTAs of the cluster arrive on.
-__device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity,
-                                                 volatile int* abort_flag, int* status) {
-    if (mbar_try_wait_cluster(bar, parity)) return true;
-    if (*abort_flag) return false;
-    const long long t0 = clock64();
-    while (!mbar_try_wait_cluster(bar, parity)) {
-        if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitCycles) {
-            *abort_flag = 1;
-            report(status, ESTP_ERR_TIMEOUT);
-            return false;
-        }
-    }
-    return true;
-}
-
-__device__ __forceinline__ void drain_wait_cluster(uint64_t* bar, uint32_t parity, int* status) {
-    const long long t0 = clock64();
-    while (!mbar_try_wait_cluster(bar, parity)) {
-        if (clock64() - t0 > kWaitCycles) {
-            report(status, ESTP_ERR_TIMEOUT);
-            return;
-        }
-    }
-}
-
-__device__ __forceinline__ bool warp_wait_cluster(uint64_t* bar, uint32_t parity,
-                                                  volatile int* abort_flag, int* status) {
-    bool r = false;
-    if ((threadIdx.x & 31) == 0) r = wait_bar_cluster(bar, parity, abort_flag, status);
-    r = __shfl_sync(0xffffffffu, r ? 1 : 0, 0) != 0;
-    __syncwarp();
-    return r;
-}
-
-// Every thread of every CTA of the cluster; all threads of a warp together.
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
-                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-}  // namespace estp

@@ -1,0 +1,55 @@
+"""Failure detection on the GPU: a bounded wait that runs out (no fault, no hang).
+
+estp_set_wait_limit lowers the limit of the tensor-core attention kernels' abortable
+waits to a few cycles, far below the latency of a tile copy, so they expire in every
+CTA.  The call must then report ESTP_ERR_TIMEOUT through estp_sync_status (the kernels
+drain the copies and MMAs they issued and free their tensor memory), and the next
+normal call on the same context must match the oracle."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from gpu_util import assert_importance
+from synth import device as sd
+from synth import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+WL = W.Workload("timeout", seed=21, B=3, T_lo=200, T_hi=900, dtype=synth.BF16, V=8,
+                n_layers_model=1, layers_used=1, Hq=8, Hkv=2, d=128, D=64, sinks=2)
+
+
+def _oracle_S(w):
+    cu = w.cu_seqlens()
+    Q, K = W.host_qk(w, w.layers[0])
+    C = oracle.attn_colsum(Q, K, cu, w.scale)
+    return oracle.importance(C, cu, 1, w.Hq)
+
+
+@pytest.mark.parametrize("lse_given", [False, True], ids=["lse_computed", "lse_given"])
+def test_wait_runs_out_then_context_recovers(cuda_lib, lse_given):
+    w = WL
+    cu = w.cu_seqlens()
+    sumT, maxT = int(cu[-1]), int(np.diff(cu).max())
+    Q, K = sd.qk(w, w.layers[0])
+    cu_d = sd.cu_seqlens(w)
+    ctx = cuda_lib.Context(0)
+    lse = ctx.attn_lse(Q, K, cu_d, maxT) if lse_given else None
+    ctx.sync_status()
+    ctx.set_wait_limit(2)
+    ctx.attn_importance(Q, K, cu_d, maxT, lse=lse)  # the row normalisers too when lse is None
+    with pytest.raises(cuda_lib.EstpError) as err:
+        ctx.sync_status()
+    assert err.value.status == cuda_lib.ESTP_ERR_TIMEOUT
+    ctx.sync_status()  # the status word was cleared by the read
+    ctx.set_wait_limit(0)
+    ctx.attn_importance(Q, K, cu_d, maxT, lse=lse)
+    S = ctx.attn_importance_finalize(1, sumT).cpu().numpy()
+    ctx.sync_status()
+    assert_importance(S, _oracle_S(w))
+    ctx.close()
+
+
+def test_wait_limit_rejects_null_context(cuda_lib):
+    assert cuda_lib.lib.estp_set_wait_limit(None, 5) == cuda_lib.ESTP_ERR_INVALID_ARG
