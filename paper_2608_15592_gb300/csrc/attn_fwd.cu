@@ -25,9 +25,10 @@
 //               a slot frees when its S is done) and V (a ring of 2, a slot frees when
 //               its P V is done)
 //   warp 1      issues S = Q K^T (as soon as a K tile and an S buffer are free)
-//   warp 2      issues O += P V (as soon as the epilogue has written P): two issuing
-//               threads, because one thread that issues 16 MMAs, makes 4 barrier checks
-//               and 5 commits per tile takes longer than the tensor pipe needs for them
+//   warp 2      issues O += P V (as soon as the epilogue has written P).  S and P V have
+//               one issuing thread each (lane 0 of warps 1 and 2), because one thread
+//               that issues 16 MMAs, makes 4 barrier checks and 5 commits per tile takes
+//               longer than the tensor pipe needs for them
 //   warps 3-18  epilogue, two groups of 8 that take the even and the odd key-tile steps
 //               (each S / P buffer belongs to one group); warp w reads TMEM lanes
 //               32 (w % 4) .. (one query row each) and one 64-column half: P, the column
@@ -179,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* q_empty = q_full + kQBufs;             // [kQBufs]
     uint64_t* k_full = q_empty + kQBufs;             // [kKStages]
     uint64_t* k_empty = k_full + kKStages;           // [kKStages]
-    uint64_t* v_full = k_empty + kKStages;           // [2] (a V^T slot is free when p_empty completes)
+    uint64_t* v_full = k_empty + kKStages;           // [2] (a V slot is free when p_empty completes)
     uint64_t* s_full = v_full + 2;                   // [2]
     uint64_t* s_empty = s_full + 2;                  // [2]
     uint64_t* p_full = s_empty + 2;                  // [2]
@@ -240,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // the plans, V^T (and the lse values) are complete past this point
+    // the plans (and the lse values) are complete past this point
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int total = a.info->ok && a.info2->ok ? a.info->total : 0;
@@ -277,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             auto load_v = [&](const VLoad& v) -> bool {
                 const int stage = (int)(v.step & 1);
                 const uint32_t u = v.step >> 1;
-                // P V of step - 2 is complete (p_empty completes with it): its V^T slot is free
+                // P V of step - 2 is complete (p_empty completes with it): its V slot is free
                 if (u >= 1 && !wait_bar(&p_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
                 mbar_expect_tx(&v_full[stage], kTileBytes);
                 for (int at = 0; at < 2; ++at)
@@ -383,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 2) {
         // ----------------------------------------------------------- PV issuer
-        // O += P(s) V(s): P from TMEM, V^T's key tile from the ring; the first tile of an
+        // O += P(s) V(s): P from TMEM, the key tile of V from its ring; the first tile of an
         // item overwrites O (once the epilogue has read the previous item's O), the last
         // one hands O to the epilogue group that takes its parity
         if (lane == 0) {
@@ -408,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
                                sw128_mn_desc(va + kk * 16 * 128),  // keys 16 kk ..
                                (kt == 0 && kk == 0) ? 0u : 1u);
-                    mma_commit(&p_empty[pb]);  // also frees the V^T slot for the producer
+                    mma_commit(&p_empty[pb]);  // also frees the V slot for the producer
                     if (kt == t.qt) mma_commit(&o_full[pb]);
                 }
             }
