@@ -50,7 +50,9 @@ typedef enum {
     ESTP_ERR_UNSUPPORTED = 2,  /* valid request the library does not implement   */
     ESTP_ERR_CUDA = 3,         /* a CUDA runtime call failed (message in last_error) */
     ESTP_ERR_TIMEOUT = 4,      /* a device-side bounded wait gave up               */
-    ESTP_ERR_WORKSPACE = 5     /* workspace could not be (re)allocated             */
+    ESTP_ERR_WORKSPACE = 5,    /* workspace could not be (re)allocated             */
+    ESTP_ERR_BOUNDS = 6        /* a device bounds check failed; only libraries built
+                                  with -DESTP_CHECKS make these checks           */
 } estp_status;
 
 typedef enum { ESTP_F32 = 0, ESTP_BF16 = 1 } estp_dtype;

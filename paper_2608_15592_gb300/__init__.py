@@ -23,9 +23,12 @@ from dataclasses import dataclass
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libestp.so")
+# the same library built with -DESTP_CHECKS (device bounds checks), for tests and debugging
+CHECKS_LIB_PATH = os.path.join(_HERE, "_build_checks", "libestp_checks.so")
 
 ESTP_OK, ESTP_ERR_INVALID_ARG, ESTP_ERR_UNSUPPORTED = 0, 1, 2
 ESTP_ERR_CUDA, ESTP_ERR_TIMEOUT, ESTP_ERR_WORKSPACE = 3, 4, 5
+ESTP_ERR_BOUNDS = 6
 ESTP_F32, ESTP_BF16 = 0, 1
 ESTP_IMP_EXCLUDE_SELF = 1
 ESTP_IMP_DIV_CAUSAL = 2
@@ -69,11 +72,13 @@ class _MlpGrads(ctypes.Structure):
                 ("b2", ctypes.c_void_p), ("pooled", ctypes.c_void_p)]
 
 
-def _load():
-    if not os.path.exists(LIB_PATH):
-        raise ImportError(f"ESTP CUDA library not built ({LIB_PATH} missing): run "
+def load_library(path: str = LIB_PATH):
+    """ctypes handle of a build of the C ABI with every entry point's signature set:
+    libestp.so by default, or CHECKS_LIB_PATH for the bounds-checked build."""
+    if not os.path.exists(path):
+        raise ImportError(f"ESTP CUDA library not built ({path} missing): run "
                           "paper_2608_15592_gb300/build.py or __graft_entry__.build()")
-    lib = ctypes.CDLL(LIB_PATH)
+    lib = ctypes.CDLL(path)
     P, I32, I64, F, U32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float,
                            ctypes.c_uint32)
     sigs = {
@@ -110,7 +115,7 @@ def _load():
     return lib
 
 
-lib = _load()
+lib = load_library()
 
 
 def _check(status: int):
@@ -157,17 +162,23 @@ class MlpHead:
 
 
 class Context:
-    """One estp_ctx (status word + workspace) on a CUDA device."""
+    """One estp_ctx (status word + workspace) on a CUDA device, in `library` (the release
+    build by default; load_library(CHECKS_LIB_PATH) for the bounds-checked one)."""
 
-    def __init__(self, device: int = 0):
+    def __init__(self, device: int = 0, library=None):
         self.device = device
+        self._lib = lib if library is None else library
         h = ctypes.c_void_p()
-        _check(lib.estp_create(ctypes.byref(h), device))
+        self._check(self._lib.estp_create(ctypes.byref(h), device))
         self._h = h
+
+    def _check(self, status: int):
+        if status != ESTP_OK:
+            raise EstpError(status, self._lib.estp_last_error(None).decode())
 
     def close(self):
         if getattr(self, "_h", None):
-            lib.estp_destroy(self._h)
+            self._lib.estp_destroy(self._h)
             self._h = None
 
     def __del__(self):
@@ -178,12 +189,12 @@ class Context:
 
     def sync_status(self, stream=None):
         """estp_sync_status: synchronise the stream; raise on a device-side error."""
-        _check(lib.estp_sync_status(self._h, _stream(stream)))
+        self._check(self._lib.estp_sync_status(self._h, _stream(stream)))
 
     def set_wait_limit(self, cycles: int = 0):
         """estp_set_wait_limit: limit (SM cycles) of the attention kernels' abortable
         waits for later calls; 0 restores the default.  A testing aid."""
-        _check(lib.estp_set_wait_limit(self._h, int(cycles)))
+        self._check(self._lib.estp_set_wait_limit(self._h, int(cycles)))
 
     # ------------------------------------------------------------------ (a)
     def lm_head_entropy(self, hidden, W, out=None, stream=None):
@@ -199,7 +210,7 @@ class Context:
         ldh = hidden.stride(0) if rows > 1 else D
         ldw = W.stride(0) if V > 1 else D
         out = torch.empty(rows, dtype=torch.float32, device=hidden.device) if out is None else out
-        _check(lib.estp_lm_head_entropy(self._h, _ptr(hidden), ldh, _ptr(W), ldw, _dtype(hidden),
+        self._check(self._lib.estp_lm_head_entropy(self._h, _ptr(hidden), ldh, _ptr(W), ldw, _dtype(hidden),
                                         rows, D, V, _ptr(out), _stream(stream)))
         return out
 
@@ -212,7 +223,7 @@ class Context:
         V = logits.shape[1] if V is None else V
         out = torch.empty(rows, dtype=torch.float32, device=logits.device) if out is None else out
         B = 0 if cu_seqlens is None else cu_seqlens.numel() - 1
-        _check(lib.estp_token_entropy(self._h, _ptr(logits), _dtype(logits), rows, V, ld,
+        self._check(self._lib.estp_token_entropy(self._h, _ptr(logits), _dtype(logits), rows, V, ld,
                                       _ptr(cu_seqlens), B, _ptr(out), _stream(stream)))
         return out
 
@@ -225,7 +236,7 @@ class Context:
         Hkv = K.shape[1]
         scale = 1.0 / math.sqrt(d) if scale is None else scale
         out = torch.empty(Hq, sumT, dtype=torch.float32, device=Q.device) if out is None else out
-        _check(lib.estp_attn_lse(self._h, _ptr(Q), _ptr(K), _dtype(Q), Hq, Hkv, d, scale,
+        self._check(self._lib.estp_attn_lse(self._h, _ptr(Q), _ptr(K), _dtype(Q), Hq, Hkv, d, scale,
                                  _ptr(cu_seqlens), cu_seqlens.numel() - 1, sumT, max_seqlen,
                                  _ptr(out), _stream(stream)))
         return out
@@ -244,7 +255,7 @@ class Context:
         else:
             arr = (ctypes.c_int32 * len(heads))(*[int(h) for h in heads])
             hp, nh = ctypes.cast(arr, ctypes.c_void_p), len(heads)
-        _check(lib.estp_attn_importance(self._h, _ptr(Q), _ptr(K), _dtype(Q), _ptr(lse), Hq,
+        self._check(self._lib.estp_attn_importance(self._h, _ptr(Q), _ptr(K), _dtype(Q), _ptr(lse), Hq,
                                         Hkv, d, scale, hp, nh, _ptr(cu_seqlens),
                                         cu_seqlens.numel() - 1, sumT, max_seqlen,
                                         1 if accumulate else 0,
@@ -265,7 +276,7 @@ class Context:
         scale = 1.0 / math.sqrt(d) if scale is None else scale
         if out is None:
             out = torch.empty(sumT, Hq, d, dtype=Q.dtype, device=Q.device)
-        _check(lib.estp_attn_forward_importance(
+        self._check(self._lib.estp_attn_forward_importance(
             self._h, _ptr(Q), _ptr(K), _ptr(V), _dtype(Q), _ptr(lse), Hq, Hkv, d, scale,
             _ptr(cu_seqlens), cu_seqlens.numel() - 1, sumT, max_seqlen, 1 if accumulate else 0,
             (ESTP_IMP_EXCLUDE_SELF if exclude_self else 0) | _DIVISOR_FLAGS[divisor], _ptr(out),
@@ -279,7 +290,7 @@ class Context:
         if out is None:
             out = torch.empty(sumT, dtype=torch.float32,
                               device=device if device is not None else f"cuda:{self.device}")
-        _check(lib.estp_attn_importance_finalize(self._h, n_layers, _ptr(out), _stream(stream)))
+        self._check(self._lib.estp_attn_importance_finalize(self._h, n_layers, _ptr(out), _stream(stream)))
         return out
 
     # ------------------------------------------------------------------ (c)
@@ -289,7 +300,7 @@ class Context:
         import torch
         B = cu_seqlens.numel() - 1
         out = torch.empty(B, 3, dtype=torch.int32, device=entropy.device) if out is None else out
-        _check(lib.estp_misalignment(self._h, _ptr(entropy), _ptr(importance), _ptr(cu_seqlens),
+        self._check(self._lib.estp_misalignment(self._h, _ptr(entropy), _ptr(importance), _ptr(cu_seqlens),
                                      B, entropy.numel(), pct, _ptr(out), _stream(stream)))
         return out
 
@@ -306,7 +317,7 @@ class Context:
         gb = torch.empty(K, dtype=torch.float32, device=dev) if grads else None
         gp = torch.empty(B, D, dtype=torch.float32, device=dev) if grads else None
         hp = ctypes.pointer(_Head(_ptr(head.W), _ptr(head.bias), _ptr(head.centers), K))
-        _check(lib.estp_head_loss(self._h, _ptr(pooled), B, D, hp, _ptr(targets), lambda3,
+        self._check(self._lib.estp_head_loss(self._h, _ptr(pooled), B, D, hp, _ptr(targets), lambda3,
                                   _ptr(loss), _ptr(gW), _ptr(gb), _ptr(gp), _stream(stream)))
         return (loss, gW, gb, gp) if grads else loss
 
@@ -321,7 +332,7 @@ class Context:
         B, D = pooled.shape
         pred = torch.empty(B, dtype=torch.float32, device=pooled.device)
         p = torch.empty(B, head.W2.shape[0], dtype=torch.float32, device=pooled.device) if probs else None
-        _check(lib.estp_mlp_head_predict(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(pred),
+        self._check(self._lib.estp_mlp_head_predict(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(pred),
                                          _ptr(p), _stream(stream)))
         return (pred, p) if probs else pred
 
@@ -340,7 +351,7 @@ class Context:
                for k, v in shapes.items()}
         loss = torch.empty(1, dtype=torch.float32, device=dev)
         gp = ctypes.pointer(_MlpGrads(*[_ptr(out[k]) for k in ("W1", "b1", "W2", "b2", "pooled")]))
-        _check(lib.estp_mlp_head_loss(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(targets),
+        self._check(self._lib.estp_mlp_head_loss(self._h, _ptr(pooled), B, D, self._mlp(head), _ptr(targets),
                                       lambda3, _ptr(loss), gp if want else None, _stream(stream)))
         if not grads:
             return loss
@@ -364,7 +375,7 @@ class Context:
             hp = ctypes.pointer(_Head(_ptr(head.W), _ptr(head.bias), _ptr(head.centers),
                                       head.W.shape[0]))
         mix = MixParams(lambda1, lambda2, alpha)
-        _check(lib.estp_pool(self._h, _ptr(hidden), _dtype(hidden), D, ldh, _ptr(entropy),
+        self._check(self._lib.estp_pool(self._h, _ptr(hidden), _dtype(hidden), D, ldh, _ptr(entropy),
                              _ptr(importance), _ptr(cu_seqlens), B, sumT, mix, hp,
                              _ptr(pooled), _ptr(pred) if head is not None else None,
                              _stream(stream)))

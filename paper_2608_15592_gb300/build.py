@@ -39,8 +39,8 @@ def _deps_mtime() -> float:
     return max(os.path.getmtime(f) for f in files)
 
 
-def _compile(src: str, extra: list[str]) -> tuple[str, str]:
-    obj = os.path.join(OUT, os.path.basename(src).replace(".cu", ".o"))
+def _compile(src: str, extra: list[str], out: str = OUT) -> tuple[str, str]:
+    obj = os.path.join(out, os.path.basename(src).replace(".cu", ".o"))
     cmd = [_nvcc(), *ARCH, *NVCC_FLAGS, *extra, "-c", src, "-o", obj]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
@@ -48,31 +48,43 @@ def _compile(src: str, extra: list[str]) -> tuple[str, str]:
     return obj, r.stderr
 
 
-def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None) -> str:
-    """Compile every csrc/*.cu for sm_103a and link libestp.so; returns its path."""
-    os.makedirs(OUT, exist_ok=True)
+OUT_CHECKS = os.path.join(PKG, "_build_checks")
+LIB_CHECKS = os.path.join(OUT_CHECKS, "libestp_checks.so")
+
+
+def build_checks(force: bool = False) -> str:
+    """The debug variant: the same sources with -DESTP_CHECKS (device bounds checks that
+    record ESTP_ERR_BOUNDS in the status word), linked as libestp_checks.so."""
+    return build(force=force, extra=["-DESTP_CHECKS"], out=OUT_CHECKS, lib=LIB_CHECKS)
+
+
+def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None,
+          out: str = OUT, lib: str = LIB) -> str:
+    """Compile every csrc/*.cu for sm_103a into `out` and link `lib` (libestp.so by
+    default); returns the library's path."""
+    os.makedirs(out, exist_ok=True)
     extra = list(extra or [])
     dep = _deps_mtime()
     srcs = _sources()
     todo = []
     for s in srcs:
-        obj = os.path.join(OUT, os.path.basename(s).replace(".cu", ".o"))
+        obj = os.path.join(out, os.path.basename(s).replace(".cu", ".o"))
         if force or not os.path.exists(obj) or os.path.getmtime(obj) < max(dep, os.path.getmtime(s)):
             todo.append(s)
     if todo:
         with cf.ThreadPoolExecutor(max_workers=min(len(todo), os.cpu_count() or 4)) as ex:
-            for obj, log in ex.map(lambda s: _compile(s, extra), todo):
+            for obj, log in ex.map(lambda s: _compile(s, extra, out), todo):
                 if verbose and log.strip():
                     print(log)
-    objs = [os.path.join(OUT, os.path.basename(s).replace(".cu", ".o")) for s in srcs]
-    if todo or not os.path.exists(LIB) or os.path.getmtime(LIB) < max(os.path.getmtime(o) for o in objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    objs = [os.path.join(out, os.path.basename(s).replace(".cu", ".o")) for s in srcs]
+    if todo or not os.path.exists(lib) or os.path.getmtime(lib) < max(os.path.getmtime(o) for o in objs):
+        tmp = lib + f".tmp{os.getpid()}"
         cmd = [_nvcc(), *ARCH, "-shared", "-o", tmp, *objs]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 def build_synth(force: bool = False) -> str:

@@ -94,6 +94,7 @@ struct FwdArgs {
     const float* lse;       // [Hq, sumT] natural log
     __nv_bfloat16* O;       // [sumT, Hq, 128]
     float* part;            // [slots][128]
+    int64_t n_slots;        // slots of part (bounds checks of debug builds)
     int* status;
 };
 
@@ -439,7 +440,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(&cs_empty[sb]);
                 const float4 sum = make_float4((x0.x + x1.x) + (x2.x + x3.x), (x0.y + x1.y) + (x2.y + x3.y),
                                                (x0.z + x1.z) + (x2.z + x3.z), (x0.w + x1.w) + (x2.w + x3.w));
-                reinterpret_cast<float4*>(a.part + (t.slot0 + kt) * kT)[lane] = sum;
+                if (in_bounds(t.slot0 + kt >= 0 && t.slot0 + kt < a.n_slots, a.status))
+                    reinterpret_cast<float4*>(a.part + (t.slot0 + kt) * kT)[lane] = sum;
             }
         }
     } else {
@@ -562,7 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 float v[32];
                 tmem_ld32(lane_base + kColO + half * 64 + ch * 32, v);
                 tmem_wait_ld();
-                if (valid) {
+                if (valid && in_bounds(t.t0 + i_loc < a.sumT && t.h >= 0 && t.h < a.Hq, a.status)) {
                     uint4* out = reinterpret_cast<uint4*>(
                         a.O + ((t.t0 + i_loc) * a.Hq + t.h) * (int64_t)kD + half * 64 + ch * 32);
 #pragma unroll
@@ -592,7 +594,7 @@ constexpr int kRedHeadLanes = 8;
 __global__ void __launch_bounds__(32 * kRedHeadLanes)
     imp_fwd_reduce_kernel(const float* __restrict__ part, const int32_t* cu, const int32_t* base2,
                           const PlanInfo* info, const PlanInfo* info2, int B, int Hq, int64_t sumT,
-                          int accumulate, float* acc) {
+                          int accumulate, float* acc, int64_t n_slots, int* status) {
     __shared__ float red[kRedHeadLanes][32];
     asm volatile("griddepcontrol.wait;" ::: "memory");  // the forward's partial slots are complete
     const int jj = threadIdx.x & 31, hl = threadIdx.x >> 5;
@@ -603,7 +605,8 @@ __global__ void __launch_bounds__(32 * kRedHeadLanes)
         const int T = cu[b + 1] - cu[b];
         const int nt = (T + kT - 1) / kT;
         const int jl = (int)(j - cu[b]), kt = jl / kT, col = jl - kt * kT;
-        for (int h = hl; h < Hq; h += kRedHeadLanes) {
+        const bool ok = in_bounds(b >= 0 && b < B && base2[b] + (int64_t)Hq * tri(nt) <= n_slots, status);
+        for (int h = hl; ok && h < Hq; h += kRedHeadLanes) {
             const int64_t s0 = base2[b] + (int64_t)h * tri(nt);
             float vh = 0.f;
             constexpr int kBatch = 8;  // loads in flight before they are added, in order
@@ -713,6 +716,7 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     a.scale_log2 = scale * kLog2e;
     a.exclude_self = exclude_self ? 1 : 0;
     a.lse = lse; a.O = static_cast<__nv_bfloat16*>(O); a.part = part; a.status = ctx->status;
+    a.n_slots = slots_bound;
     e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward smem attribute");
     cudaLaunchConfig_t cf = config(dim3((unsigned)ctx->num_sms), dim3(kThreads), kSmemBytes);
@@ -720,7 +724,8 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     if (e != cudaSuccess) return cuda_fail(e, "attention forward launch");
     cudaLaunchConfig_t cr = config(dim3((unsigned)((sumT + 31) / 32)), dim3(32 * kRedHeadLanes), 0);
     e = cudaLaunchKernelEx(&cr, imp_fwd_reduce_kernel, (const float*)part, cu, (const int32_t*)base2,
-                           (const PlanInfo*)info, (const PlanInfo*)info2, B, Hq, sumT, accumulate ? 1 : 0, acc);
+                           (const PlanInfo*)info, (const PlanInfo*)info2, B, Hq, sumT, accumulate ? 1 : 0, acc,
+                           slots_bound, ctx->status);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward reduce launch");
     e = cudaGetLastError();
     return e == cudaSuccess ? ESTP_OK : cuda_fail(e, "attention forward reduce launch");

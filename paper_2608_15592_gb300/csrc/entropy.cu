@@ -37,6 +37,7 @@ struct EntArgs {
     int64_t n_warps;
     float* H;
     EntPart* part;      // [n_warps][2]: slot 0 = first segment, slot 1 = last segment
+    int* status;        // device status word, or nullptr (bounds checks of debug builds)
 };
 
 __device__ __forceinline__ int64_t warp_start(int64_t units, int64_t W, int64_t w) {
@@ -216,6 +217,8 @@ __global__ void __launch_bounds__(kEntThreads, kEntMinBlocks) entropy_kernel(Ent
         const int64_t row_u0 = r * a.nvec;
         const int64_t seg_end = min(end, row_u0 + a.nvec);
         const int64_t c0 = u - row_u0, c1 = seg_end - row_u0;
+        if (!in_bounds(r < a.units / a.nvec && c0 >= 0 && c0 < c1 && c1 <= a.nvec, a.status))
+            return;
         float m = kMaskedLogit;
         float2 s = make_float2(0.f, 0.f), t = make_float2(0.f, 0.f);
         segment<kBf16>(a.base + r * a.ld_bytes, c0, c1, a.nvec, tail_valid, m, s, t);
@@ -230,7 +233,7 @@ __global__ void __launch_bounds__(kEntThreads, kEntMinBlocks) entropy_kernel(Ent
         if (lane == 0) {
             if (c0 == 0 && c1 == a.nvec) {
                 a.H[r] = entropy_of(ss, tt);
-            } else {
+            } else if (in_bounds(w < a.n_warps, a.status)) {
                 a.part[w * 2 + (u == start ? 0 : 1)] = EntPart{m, ss, tt, 0.f};
             }
         }
@@ -251,6 +254,7 @@ __global__ void entropy_merge_kernel(EntArgs a, int64_t n_rows, const int32_t* c
     for (int64_t w = w_lo; w <= w_hi; ++w) {
         const int64_t st = warp_start(a.units, a.n_warps, w);
         if (st == warp_start(a.units, a.n_warps, w + 1)) continue;  // empty range
+        if (!in_bounds(w >= 0 && w < a.n_warps, status)) return;
         const EntPart p = a.part[w * 2 + (st / a.nvec == r ? 0 : 1)];
         merge(m, s, t, p.m, p.s, p.t);
     }
@@ -279,6 +283,7 @@ estp_status launch_entropy(estp_ctx* ctx, const void* logits, estp_dtype dtype, 
     if (s != ESTP_OK) return s;
     a.part = static_cast<EntPart*>(ctx->ws);
     a.H = H;
+    a.status = ctx->status;
     const int64_t blocks = (a.n_warps + kEntThreads / 32 - 1) / (kEntThreads / 32);
     if (dtype == ESTP_BF16) entropy_kernel<true><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
     else entropy_kernel<false><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
@@ -354,6 +359,7 @@ estp_status launch_entropy_noalloc(const void* logits, estp_dtype dtype, int64_t
     a.n_warps = a.units < max_warps ? a.units : max_warps;
     a.part = d.part;
     a.H = H;
+    a.status = nullptr;
     const int64_t blocks = (a.n_warps + kEntThreads / 32 - 1) / (kEntThreads / 32);
     if (dtype == ESTP_BF16) entropy_kernel<true><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);
     else entropy_kernel<false><<<(unsigned)blocks, kEntThreads, 0, st>>>(a);

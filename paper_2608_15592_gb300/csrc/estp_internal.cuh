@@ -58,6 +58,20 @@ inline int esize(estp_dtype t) { return t == ESTP_BF16 ? 2 : 4; }
 // --------------------------------------------------------------- device helpers
 __device__ __forceinline__ void report(int* status, int code) { atomicCAS(status, 0, code); }
 
+// Debug builds (-DESTP_CHECKS): bounds checks on the kernels' global accesses.  A failed
+// check records ESTP_ERR_BOUNDS in the status word (when the launch has one) and the
+// caller skips the access; nothing traps.  Release builds compile the checks away.
+__device__ __forceinline__ bool in_bounds(bool ok, int* status) {
+#ifdef ESTP_CHECKS
+    if (!ok && status != nullptr) report(status, ESTP_ERR_BOUNDS);
+    return ok;
+#else
+    (void)ok;
+    (void)status;
+    return true;
+#endif
+}
+
 // 16-byte streaming load that bypasses L1 (data read exactly once).
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
     uint4 v;

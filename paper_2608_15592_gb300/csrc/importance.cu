@@ -112,6 +112,8 @@ struct SimtArgs {
     int exclude_self;
     float* part;               // [c_max][n_groups][sumT]
     float* lse_out;            // LSE kernel output [Hq, sumT]
+    int c_max;                 // chunk slots of part (bounds checks of debug builds)
+    int* status;
 };
 
 // Rows [row0, row0 + n) of a [rows, heads, d] tensor, head h, into smem as fp32
@@ -269,6 +271,7 @@ __global__ void __launch_bounds__(kSThreads) imp_simt_kernel(SimtArgs a) {
             }
         }
         const int c_slot = (it.qt0 - it.kt) / kSQc;
+        if (!in_bounds(c_slot >= 0 && c_slot < a.c_max, a.status)) continue;
         float* out = a.part + ((int64_t)c_slot * a.hs.n_groups + it.g) * a.sumT + it.t0;
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
@@ -293,7 +296,7 @@ __device__ __forceinline__ const int32_t* stage_cu(const int32_t* cu, int B, int
 
 __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const int32_t* cu,
                                   int B, int64_t sumT, int n_groups, int tile, int qc,
-                                  int accumulate, float* acc) {
+                                  int accumulate, float* acc, int c_max, int* status) {
     __shared__ int32_t cu_s[kCuStage];
     const int32_t* cuv = stage_cu(cu, B, cu_s);
     // the partials are complete past this point (launched as a programmatic dependent
@@ -307,7 +310,8 @@ __global__ void imp_reduce_kernel(const float* part, const PlanInfo* info, const
         const int T = cuv[b + 1] - cuv[b];
         const int nt = (T + tile - 1) / tile;
         const int kt = (int)((j - cuv[b]) / tile);
-        const int n = chunks_of(nt, kt, qc) * n_groups;  // partials (c, g), c-major
+        int n = chunks_of(nt, kt, qc) * n_groups;  // partials (c, g), c-major
+        if (!in_bounds(n <= c_max * n_groups && b >= 0 && b < B, status)) n = 0;
         // up to 16 partials are loaded before any is added (independent loads in flight),
         // then added in the same (c, g) order
         constexpr int kBatch = 16;
@@ -333,6 +337,7 @@ __global__ void imp_finalize_kernel(const float* acc, const int32_t* cu, int B, 
     const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= sumT) return;
     const int b = upper_slot(cuv, B, j);
+    if (!in_bounds(b >= 0 && b < B, nullptr)) return;
     int64_t n = cuv[b + 1] - cuv[b];
     if (div == 1) n = (int64_t)cuv[b + 1] - j - (exclude_self ? 1 : 0);
     else if (div == 2) n = 1;
@@ -436,13 +441,14 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
                                          info, ctx->status);
     if (tc) {
         s = launch_imp_tc(ctx, Q, K, lse_use, Hq, Hkv, d, scale, hs, cu, B, sumT,
-                          (flags & ESTP_IMP_EXCLUDE_SELF) != 0, base, info, part, st);
+                          (flags & ESTP_IMP_EXCLUDE_SELF) != 0, base, info, part, c_max, st);
         if (s != ESTP_OK) return s;
     } else {
         SimtArgs a{};
         a.Q = Q; a.K = K; a.lse = lse_use; a.cu = cu; a.base = base; a.info = info; a.B = B;
         a.Hq = Hq; a.Hkv = Hkv; a.d = d; a.sumT = sumT; a.scale_log2 = scale * kLog2e;
         a.hs = hs; a.exclude_self = (flags & ESTP_IMP_EXCLUDE_SELF) != 0; a.part = part;
+        a.c_max = c_max; a.status = ctx->status;
         const size_t smem = simt_smem(d, true);
         const void* kfn = dtype == ESTP_BF16 ? (const void*)imp_simt_kernel<true> : (const void*)imp_simt_kernel<false>;
         cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -462,7 +468,7 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
         cfg.numAttrs = 1;
         cudaError_t e = cudaLaunchKernelEx(&cfg, imp_reduce_kernel, (const float*)part,
                                            (const PlanInfo*)info, cu, B, sumT, hs.n_groups, tile,
-                                           qc, accumulate ? 1 : 0, acc);
+                                           qc, accumulate ? 1 : 0, acc, c_max, ctx->status);
         if (e != cudaSuccess) return cuda_fail(e, "importance reduce launch");
     }
     cudaError_t e = cudaGetLastError();

@@ -98,6 +98,7 @@ struct TcArgs {
     float* lse_out;     // LSE mode output [Hq, sumT]
     int* status;
     long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
+    int c_max;              // column-sum mode: chunk slots of the partial buffer (bounds checks)
     ImpHeads hs;
 };
 
@@ -326,6 +327,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             break;
                         }
                         const int64_t x = (int64_t)head * a.sumT + t.t0 + row0;
+                        if (!in_bounds(x >= 0 && x < (int64_t)a.Hq * a.sumT, a.status)) {
+                            *abort_flag = 1;  // the consumers leave at their next wait
+                            ok = false;
+                            break;
+                        }
                         mbar_expect_tx(&lse_full[ls], kLseBox * 4);
                         tma_load_1d(lse_ring + ls * (kLseSlotBytes / 4), &tm_lse, (int)(x & ~int64_t(3)),
                                     &lse_full[ls]);
@@ -564,14 +570,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(xe);
                 if (MODE == kModeImp) {
                     const int j = t.fix_row0 + tau * kTile + row;
-                    if (j < t.T)
+                    if (j < t.T && in_bounds(t.chunk >= 0 && t.chunk < a.c_max && t.g >= 0 &&
+                                                 t.g < a.hs.n_groups && t.t0 + j < a.sumT,
+                                             a.status))
                         a.part[((int64_t)t.chunk * a.hs.n_groups + t.g) * a.sumT + t.t0 + j] =
                             acc2.x + acc2.y + o.x;
                 } else {
                     const float mm = fmaxf(m, o.x);
                     const float ss = ssum * ex2(m - mm) + o.y * ex2(o.x - mm);
                     const int i = t.fix_row0 + tau * kTile + row;
-                    if (i < t.T) a.lse_out[(int64_t)t.h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
+                    if (i < t.T && in_bounds(t.h >= 0 && t.h < a.Hq && t.t0 + i < a.sumT, a.status))
+                        a.lse_out[(int64_t)t.h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
                 }
             }
         }
@@ -680,8 +689,9 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
 estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const float* lse, int Hq,
                           int Hkv, int d, float scale, const ImpHeads& hs, const int32_t* cu,
                           int B, int64_t sumT, bool exclude_self, const int32_t* base,
-                          const PlanInfo* info, float* part, cudaStream_t st) {
+                          const PlanInfo* info, float* part, int c_max, cudaStream_t st) {
     TcArgs a{};
+    a.c_max = c_max;
     a.cu = cu; a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.sumT = sumT;
     a.base = base; a.info = info;
     a.scale_log2 = scale * kLog2e;

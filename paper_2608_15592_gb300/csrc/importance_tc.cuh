@@ -15,6 +15,6 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
 estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const float* lse, int Hq,
                           int Hkv, int d, float scale, const ImpHeads& hs, const int32_t* cu,
                           int B, int64_t sumT, bool exclude_self, const int32_t* base,
-                          const PlanInfo* info, float* part, cudaStream_t st);
+                          const PlanInfo* info, float* part, int c_max, cudaStream_t st);
 
 }  // namespace estp

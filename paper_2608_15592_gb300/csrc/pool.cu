@@ -67,6 +67,7 @@ struct FinishArgs {
     const float* centers;
     int K;
     float* pred;
+    int* status;             // bounds checks of debug builds
 };
 
 // Eight bf16 (or four fp32) values of one 16-byte unit, weighted by e, added to acc.
@@ -188,6 +189,7 @@ __global__ void __launch_bounds__(kMaxThreads, 2) pool_stream_kernel(const Strea
             __syncthreads();  // e_s is rewritten by the next window
         }
         const int slot = c + b;
+        if (!in_bounds(slot >= 0 && slot < a.G + a.B && b < a.B, a.status)) return;
         if (active) {
             float* out = a.P + (int64_t)slot * a.D + u * kPer;
             const int64_t left = a.D - u * kPer;
@@ -261,7 +263,7 @@ __global__ void __launch_bounds__(kFinThreads) pool_finish_kernel(const FinishAr
     // the stream kernel's slots are complete past this point
     asm volatile("griddepcontrol.wait;" ::: "memory");
     float2 h = make_float2(0.f, 0.f);
-    if (t1 > t0) {
+    if (t1 > t0 && in_bounds(owner_cta(t1 - 1, a.sumT, a.G) + b < a.G + a.B, a.status)) {
         const int c0 = owner_cta(t0, a.sumT, a.G), c1 = owner_cta(t1 - 1, a.sumT, a.G);
         const int n = c1 - c0 + 1;
         // (M*, Z*) in one pass: online per thread, then warps and the CTA in fixed order
@@ -432,6 +434,7 @@ estp_status launch_pool(estp_ctx* ctx, const void* hidden, estp_dtype dtype, int
     if (dtype == ESTP_BF16) pool_stream_kernel<true><<<grid, threads, 0, st>>>(a);
     else pool_stream_kernel<false><<<grid, threads, 0, st>>>(a);
     FinishArgs f{};
+    f.status = ctx->status;
     f.P = a.P;
     f.MZ = a.MZ;
     f.cu = cu;
