@@ -432,7 +432,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int item = consume_item(it, true);
             if (item < 0) break;
             const TcItem t = make_item<MODE>(a, item);
-            float2 acc2 = make_float2(0.f, 0.f);   // column-sum mode
+            // column-sum mode: partial sums of this thread's four key rows 8 s + g8 (s = 0..3)
+            // of the quarter, over its columns (16x256b layout, see below)
+            float2 acc4[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                              make_float2(0.f, 0.f)};
             float m = -1e30f, ssum = 0.f;          // LSE mode
             StepIter<MODE> si(a, t);
             auto do_step = [&](int s) -> bool {
@@ -477,7 +480,65 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t taddr =
                     tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((ab * 2 + tau) * kAccCols + col0);
                 const float2 sc = make_float2(a.scale_log2, a.scale_log2);
-                // chunks of 32 columns: load, (release the accumulator after the last), reduce
+                if constexpr (MODE == kModeImp) {
+                    // 16x256b loads: thread (g8, c4) = (lane / 4, lane % 4) holds key rows
+                    // q*32 + 16 lh + 8 jj + g8 and query columns 64 h + 8 k + 2 c4 + {0, 1}.
+                    // Each query column's -lse log2e is then needed by 8 lanes only: 8
+                    // two-float shared loads per 64 columns, each one wavefront, instead of
+                    // every lane reading all 128 values (the shared-memory pipe was the bound).
+                    const int g8 = lane >> 2, c4 = lane & 3;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        float2 n2[8];
+#pragma unroll
+                        for (int k = 0; k < 8; ++k)
+                            n2[k] = *reinterpret_cast<const float2*>(nl + h * 64 + 8 * k + 2 * c4);
+#pragma unroll
+                        for (int lh = 0; lh < 2; ++lh) {
+                            uint32_t raw[32];
+                            tmem_ld16x256_x8(taddr + ((uint32_t)(16 * lh) << 16) + (uint32_t)(h * 64), raw);
+                            tmem_wait_ld();
+                            if (h == 1 && lh == 1) {  // all 128 columns read: release the accumulator
+                                tc_fence_before();
+                                __syncwarp();
+                                if (lane == 0) mbar_arrive(&acc_empty[abar]);
+                            }
+                            if (!imp_diag) {
+#pragma unroll
+                                for (int k = 0; k < 8; ++k) {
+                                    const float2 x0 = __ffma2_rn(
+                                        make_float2(__uint_as_float(raw[4 * k]), __uint_as_float(raw[4 * k + 1])),
+                                        sc, n2[k]);
+                                    const float2 x1 = __ffma2_rn(
+                                        make_float2(__uint_as_float(raw[4 * k + 2]), __uint_as_float(raw[4 * k + 3])),
+                                        sc, n2[k]);
+                                    acc4[2 * lh] = __fadd2_rn(acc4[2 * lh], make_float2(ex2(x0.x), ex2(x0.y)));
+                                    acc4[2 * lh + 1] = __fadd2_rn(acc4[2 * lh + 1], make_float2(ex2(x1.x), ex2(x1.y)));
+                                }
+                            } else {  // diagonal tile: query i = column, key j = row; keep i >= j
+#pragma unroll
+                                for (int k = 0; k < 8; ++k) {
+#pragma unroll
+                                    for (int jj = 0; jj < 2; ++jj) {
+                                        const float2 x = __ffma2_rn(
+                                            make_float2(__uint_as_float(raw[4 * k + 2 * jj]),
+                                                        __uint_as_float(raw[4 * k + 2 * jj + 1])),
+                                            sc, n2[k]);
+                                        const int i0 = h * 64 + 8 * k + 2 * c4;
+                                        const int j = q * 32 + 16 * lh + 8 * jj + g8;
+                                        const bool k0 = a.exclude_self ? i0 > j : i0 >= j;
+                                        const bool k1 = a.exclude_self ? i0 + 1 > j : i0 + 1 >= j;
+                                        acc4[2 * lh + jj] = __fadd2_rn(
+                                            acc4[2 * lh + jj], make_float2(k0 ? ex2(x.x) : 0.f, k1 ? ex2(x.y) : 0.f));
+                                    }
+                                }
+                            }
+                        }
+                    }
+                    return true;
+                } else {
+                // LSE mode: chunks of 32 columns of this thread's query row: load, (release the
+                // accumulator after the last), reduce
 #pragma unroll
                 for (int ch = 0; ch < kChunks; ++ch) {
                     float v[32];
@@ -489,31 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (lane == 0) mbar_arrive(&acc_empty[abar]);
                     }
                     const int cb = col0 + ch * 32;  // tile column of v[0]
-                    const float* nc = nl + ch * 32;
-                    if (MODE == kModeImp) {
-                        if (!imp_diag) {
-                            float2 acc_b = make_float2(0.f, 0.f);
-#pragma unroll
-                            for (int c = 0; c < 32; c += 4) {
-                                const float4 n4 = *reinterpret_cast<const float4*>(nc + c);
-                                float2 x0 = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, make_float2(n4.x, n4.y));
-                                float2 x1 = __ffma2_rn(make_float2(v[c + 2], v[c + 3]), sc, make_float2(n4.z, n4.w));
-                                acc2 = __fadd2_rn(acc2, make_float2(ex2(x0.x), ex2(x0.y)));
-                                acc_b = __fadd2_rn(acc_b, make_float2(ex2(x1.x), ex2(x1.y)));
-                            }
-                            acc2 = __fadd2_rn(acc2, acc_b);
-                        } else {  // diagonal tile: query i = col, key j = row (local); keep i >= j
-#pragma unroll
-                            for (int c = 0; c < 32; c += 2) {
-                                const float2 n2 = *reinterpret_cast<const float2*>(nc + c);
-                                float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc, n2);
-                                const int i0 = cb + c, i1 = i0 + 1;
-                                const bool k0 = a.exclude_self ? i0 > row : i0 >= row;
-                                const bool k1 = a.exclude_self ? i1 > row : i1 >= row;
-                                acc2 = __fadd2_rn(acc2, make_float2(k0 ? ex2(x.x) : 0.f, k1 ? ex2(x.y) : 0.f));
-                            }
-                        }
-                    } else {
+                    {
                         if (lse_diag) {  // diagonal tile: keys j = col after the query i = row
 #pragma unroll
                             for (int c = 0; c < 32; ++c)
@@ -545,10 +582,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 return true;
+                }
             };
             for (int s = 0; s < t.n_steps; ++s, ++step, si.next(a, t))
                 if ((MODE == kModeLse || (int)(step & 1) == sub) && !(ok = do_step(s))) break;
             if (!ok) break;
+            // column-sum mode: the four lanes c4 of a g8 hold columns of the same four rows;
+            // a butterfly over them gives each the rows' sums (the same bits in all four,
+            // as the additions pair the same operands), and lane (g8, c4) keeps row
+            // 8 c4 + g8 of the quarter
+            int my_row = lane;  // row of the quarter this thread merges and writes
+            float my_sum = 0.f;
+            if constexpr (MODE == kModeImp) {
+                float rs[4];
+#pragma unroll
+                for (int r4 = 0; r4 < 4; ++r4) rs[r4] = acc4[r4].x + acc4[r4].y;
+#pragma unroll
+                for (int r4 = 0; r4 < 4; ++r4) {
+                    rs[r4] += __shfl_xor_sync(0xffffffffu, rs[r4], 1);
+                    rs[r4] += __shfl_xor_sync(0xffffffffu, rs[r4], 2);
+                }
+                const int c4 = lane & 3;
+                my_row = 8 * c4 + (lane >> 2);
+                my_sum = c4 == 0 ? rs[0] : c4 == 1 ? rs[1] : c4 == 2 ? rs[2] : rs[3];
+            }
             // merge the two partials of each row (bounded mbarrier hand-off), then write
             const int pb = it & 1;
             const uint32_t use = (uint32_t)(it >> 1);
@@ -558,23 +615,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (sub == 1) {
                 if (use >= 1) ok = warp_wait(xe, (use - 1) & 1, abort_flag, a.status, a.wait_cycles);
                 if (!ok) break;
-                mb[q * 32 + lane] = MODE == kModeImp ? make_float2(acc2.x + acc2.y, 0.f)
-                                                     : make_float2(m, ssum);
+                mb[q * 32 + my_row] = MODE == kModeImp ? make_float2(my_sum, 0.f) : make_float2(m, ssum);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(xf);
             } else {
                 ok = warp_wait(xf, use & 1, abort_flag, a.status, a.wait_cycles);
                 if (!ok) break;
-                const float2 o = mb[q * 32 + lane];
+                const float2 o = mb[q * 32 + my_row];
                 __syncwarp();
                 if (lane == 0) mbar_arrive(xe);
                 if (MODE == kModeImp) {
-                    const int j = t.fix_row0 + tau * kTile + row;
+                    const int j = t.fix_row0 + tau * kTile + q * 32 + my_row;
                     if (j < t.T && in_bounds(t.chunk >= 0 && t.chunk < a.c_max && t.g >= 0 &&
                                                  t.g < a.hs.n_groups && t.t0 + j < a.sumT,
                                              a.status))
                         a.part[((int64_t)t.chunk * a.hs.n_groups + t.g) * a.sumT + t.t0 + j] =
-                            acc2.x + acc2.y + o.x;
+                            my_sum + o.x;
                 } else {
                     const float mm = fmaxf(m, o.x);
                     const float ss = ssum * ex2(m - mm) + o.y * ex2(o.x - mm);

@@ -24,7 +24,8 @@ def _run(estp, library, w, dtype_q):
     sumT, maxT = int(cu[-1]), int(np.diff(cu).max())
     ctx = estp.Context(0, library=library)
     cu_d = sd.cu_seqlens(w)
-    x = sd.logits(w, 0, sumT, ld=w.V + 8, pad_val=3.0)
+    ld = (w.V + 7) // 8 * 8 + 8  # padded rows, 16-byte row stride
+    x = sd.logits(w, 0, sumT, ld=ld, pad_val=3.0)
     out = {"H": ctx.token_entropy(x, V=w.V, cu_seqlens=cu_d)}
     Q, K = sd.qk(w, w.layers[0])
     Q, K = Q.to(dtype_q), K.to(dtype_q)
@@ -46,7 +47,7 @@ def _run(estp, library, w, dtype_q):
     out["pooled"], out["pred"] = pooled, pred
     Hn = torch.full((sumT,), float("nan"), device="cuda")
     rc = library.estp_token_entropy_noalloc(ctypes.c_void_p(x.data_ptr()), estp.ESTP_BF16, sumT,
-                                            w.V, w.V + 8, ctypes.c_void_p(Hn.data_ptr()), None)
+                                            w.V, ld, ctypes.c_void_p(Hn.data_ptr()), None)
     assert rc == estp.ESTP_OK
     out["H_noalloc"] = Hn
     ctx.sync_status()  # raises EstpError(ESTP_ERR_BOUNDS) if any check fired
