@@ -399,6 +399,9 @@ def run_ours(args, rank, world, local_rank):
         "config": out_cfg, "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu,
         "e2e": e2e, "gpu_launches": lib_launches(w) * K, "clocks": clocks,
         "region_ms_per_step": region_ms / K, "calls_ms_per_step": calls_total / K,
+        # context: a prefill's flash attention returns the row normalisers, and the path
+        # then skips estp_attn_lse (the same metric without the lse calls' time)
+        "value_lse_supplied": tokens * K / ((calls_total - call_ms["lse"]) / 1e3) if world == 1 else None,
         "generator_launches_per_step": gen_per_step,
         "e2e_from_hidden": e2e_hidden,
     }
@@ -925,18 +928,50 @@ def run_reference(args, rank, world):
     }
 
 
+def _full_inputs(w):
+    """Every input of the batch on the host: drawn by the device generator and copied
+    back when a GPU is present (the same bits as the host generator, which is far slower
+    for the 3.3e9 logits of the Qwen batch), else by the host generator."""
+    import numpy as np
+    from synth import workloads as W
+    sumT = int(w.cu_seqlens()[-1])
+    try:
+        import torch
+        gpu = torch.cuda.is_available()
+    except Exception:
+        gpu = False
+    if not gpu:
+        rows = np.arange(sumT)
+        return (W.host_logits(w, rows), [W.host_qk(w, layer) for layer in w.layers],
+                W.host_hidden(w, rows))
+    import __graft_entry__
+    __graft_entry__._build_module().build_synth()  # the generator's device side only
+    from synth import device as sd
+
+    def host(t):
+        if t.dtype == torch.bfloat16:
+            return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        return t.cpu().numpy()
+
+    x = host(sd.logits(w, 0, sumT))
+    qk = []
+    for layer in w.layers:
+        Q, K = sd.qk(w, layer)
+        qk.append((host(Q), host(K)))
+    hid = host(sd.hidden(w))
+    torch.cuda.empty_cache()
+    return x, qk, hid
+
+
 def _full_oracle_step(w):
     """The oracle over the whole batch: entropy of every row, importance of every
     selected layer and head, pooling and the head."""
     import numpy as np
     import oracle
-    from synth import workloads as W
     n = os.cpu_count() or 1
     cu = w.cu_seqlens()
     sumT = int(cu[-1])
-    x = W.host_logits(w, np.arange(sumT))
-    qk = [W.host_qk(w, layer) for layer in w.layers]
-    hid = W.host_hidden(w, np.arange(sumT))
+    x, qk, hid = _full_inputs(w)
     head = w.head_params()
 
     def step():
