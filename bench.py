@@ -45,7 +45,7 @@ sys.path.insert(0, ROOT)
 METRIC = "prompt tokens/s through ESTP features (1 GB300)"
 UNIT = "tokens/s"
 DEFAULT_WORKLOAD = "llama3-8b_rl256"
-HOST_POOL_BYTES = 32 << 30   # pinned host memory the end-to-end legs may hold
+HOST_POOL_BYTES = 32 << 30   # pinned host memory the end-to-end legs may hold (per process)
 STREAM_FRACTION = 0.80       # stream Q/K per layer when resident inputs exceed this share of free HBM
 
 
@@ -418,14 +418,31 @@ class HostPool:
     input size over the host link: layer n's Q/K from pool layer n mod Lp, logit row r
     from pool row r mod R."""
 
+    @staticmethod
+    def budget() -> int:
+        """HOST_POOL_BYTES, or less: at most a third of the host's available memory shared
+        by the processes of this node (torchrun's LOCAL_WORLD_SIZE)."""
+        avail = None
+        try:
+            with open("/proc/meminfo") as f:
+                for line in f:
+                    if line.startswith("MemAvailable:"):
+                        avail = int(line.split()[1]) * 1024
+        except OSError:
+            pass
+        local = max(1, int(os.environ.get("LOCAL_WORLD_SIZE", os.environ.get("WORLD_SIZE", 1))))
+        cap = HOST_POOL_BYTES if avail is None else min(HOST_POOL_BYTES, avail // (3 * local))
+        return max(cap, 1 << 30)
+
     def __init__(self, st):
         import torch
         w = st.w
         self.st = st
+        self.bytes = self.budget()
         self.hidden = self._pin(st.hidden)
-        left = HOST_POOL_BYTES - st.hidden.numel() * st.hidden.element_size()
+        left = self.bytes - st.hidden.numel() * st.hidden.element_size()
         lb = layer_qk_bytes(w, st.sumT)
-        self.Lp = max(1, min(st.n_layers, int(0.4 * left) // lb))
+        self.Lp = max(1, min(st.n_layers, int(0.4 * max(left, 0)) // lb))
         self.q, self.k = [], []
         for n in range(self.Lp):
             Q, K = st.qk(n)
@@ -433,7 +450,7 @@ class HostPool:
             self.k.append(self._pin(K))
         left -= self.Lp * lb
         row_bytes = st.logits.shape[1] * st.logits.element_size()
-        self.R = max(1, min(st.sumT, left // row_bytes))
+        self.R = max(1, min(st.sumT, max(left, 0) // row_bytes))
         self.logits = self._pin(st.logits[:self.R])
         self.pred = torch.empty(st.pred.shape, dtype=torch.float32, pin_memory=True)
         self.pooled = torch.empty(st.pooled.shape, dtype=torch.float32, pin_memory=True)
@@ -462,7 +479,7 @@ class HostPool:
         st = self.st
         if self.R == st.sumT and self.Lp == st.n_layers:
             return "pinned host copies of every input"
-        return (f"pinned host pool of {HOST_POOL_BYTES >> 30} GiB: hidden states, Q/K of "
+        return (f"pinned host pool of {self.bytes / 2**30:.1f} GiB: hidden states, Q/K of "
                 f"{self.Lp} of {st.n_layers} layers (layer n from pool layer n mod {self.Lp}), "
                 f"{self.R} of {st.sumT} logit rows (row r from pool row r mod {self.R}); "
                 "every step copies its full input size over the host link")
