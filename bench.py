@@ -828,6 +828,25 @@ class OracleSample:
 
     PAIR_BUDGET = 6e8  # query-key pairs x heads of the importance sample
 
+    @classmethod
+    def sizing(cls, w, n_threads: int):
+        """(prompt b, heads, first query row, query-key pairs per head) of the sample."""
+        import numpy as np
+        lens = np.diff(w.cu_seqlens()).astype(np.int64)
+        b = int(np.argmin(np.abs(lens - np.median(lens))))
+        T = int(lens[b])
+        full = T * (T + 1) // 2
+        if full * w.Hq <= cls.PAIR_BUDGET:
+            h, r0 = w.Hq, 0
+        else:
+            h = min(w.Hq, n_threads)
+            # first row r0 with (T (T + 1) - r0 (r0 + 1)) / 2 pairs per head within budget
+            per_head = cls.PAIR_BUDGET / h
+            r0 = 0 if full <= per_head else int(math.ceil(
+                (-1 + math.sqrt(1 + 4 * (T * (T + 1) - 2 * per_head))) / 2))
+        heads = np.unique(np.linspace(0, w.Hq - 1, h).round().astype(np.int32))
+        return b, heads, r0, (T * (T + 1) - r0 * (r0 + 1)) / 2.0
+
     def __init__(self, w):
         import numpy as np
         from synth import workloads as W
@@ -839,21 +858,10 @@ class OracleSample:
         self.ent_rows = np.unique(np.linspace(0, self.sumT - 1, min(self.sumT, 64)).round()
                                   .astype(np.int64))
         self.x = W.host_logits(w, self.ent_rows)
-        b = int(np.argmin(np.abs(lens - np.median(lens))))
+        b, self.heads, r0, pairs = self.sizing(w, self.n_threads)
         self.rows = np.arange(cu[b], cu[b + 1])
         T = len(self.rows)
-        full = T * (T + 1) // 2
-        if full * w.Hq <= self.PAIR_BUDGET:
-            h, r0 = w.Hq, 0
-        else:
-            h = min(w.Hq, self.n_threads)
-            # first row r0 with (T (T + 1) - r0 (r0 + 1)) / 2 pairs per head within budget
-            per_head = self.PAIR_BUDGET / h
-            r0 = 0 if full <= per_head else int(math.ceil(
-                (-1 + math.sqrt(1 + 4 * (T * (T + 1) - 2 * per_head))) / 2))
-        self.heads = np.unique(np.linspace(0, w.Hq - 1, h).round().astype(np.int32))
         self.row_from = r0
-        pairs = (T * (T + 1) - r0 * (r0 + 1)) / 2.0
         # query rows before row_from are never read by the oracle: left zero
         layer = w.layers[-1]
         self.K = W.host_k(w, layer, self.rows)
