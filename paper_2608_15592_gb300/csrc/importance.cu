@@ -393,7 +393,7 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
                               cudaStream_t st) {
     const bool tc = tc_supported(dtype, d);
     const int tile = tc ? tc_tile() : kSTile;
-    const int qc = tc ? tc_qc() : kSQc;
+    const int qc = tc ? tc_qc(B, sumT, hs.n_groups, ctx->num_sms) : kSQc;
     const int nt_max = (max_seqlen + tile - 1) / tile;
     const int c_max = nt_max > 0 ? chunks_of(nt_max, 0, qc) : 0;
     // workspace: [own lse][plan base][info][partials]
@@ -441,7 +441,7 @@ estp_status launch_importance(estp_ctx* ctx, const void* Q, const void* K, estp_
                                          info, ctx->status);
     if (tc) {
         s = launch_imp_tc(ctx, Q, K, lse_use, Hq, Hkv, d, scale, hs, cu, B, sumT,
-                          (flags & ESTP_IMP_EXCLUDE_SELF) != 0, base, info, part, c_max, st);
+                          (flags & ESTP_IMP_EXCLUDE_SELF) != 0, base, info, part, c_max, qc, st);
         if (s != ESTP_OK) return s;
     } else {
         SimtArgs a{};

@@ -46,7 +46,11 @@ namespace {
 
 constexpr int kTile = 128;             // rows of a fixed or streamed tile
 constexpr int kPair = 2 * kTile;       // rows of the fixed pair (the plan's tile)
-constexpr int kQcPair = 2;             // pairs of query tiles per column-sum item
+// Pairs of query tiles per column-sum item: the largest of kQcChoices that still gives the
+// persistent grid about kItemsPerSm items per SM (tc_qc).  Longer items cost fewer item
+// hand-offs; too few items leave SMs idle at the end of a launch.
+constexpr int kQcChoices[4] = {16, 8, 4, 2};
+constexpr int kItemsPerSm = 16;
 constexpr int kEpiWarp0 = 2;           // warps 2..17
 constexpr int kEpiWarps = 16;          // 8 per fixed tile (LSE) or 4 per tile and buffer (column sums)
 // MMA issuers: warp 1 for fixed tile A, warp 18 for tile B, so that one issuer's barrier
@@ -99,6 +103,7 @@ struct TcArgs {
     int* status;
     long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
     int c_max;              // column-sum mode: chunk slots of the partial buffer (bounds checks)
+    int qc;                 // column-sum mode: pairs of query tiles per item
     ImpHeads hs;
 };
 
@@ -130,14 +135,14 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
         t.n_steps = min(t.qt0 + 2, nt);    // key tiles 0 .. the pair's last tile
         t.g = 0; t.kt = 0; t.qt1 = t.qt0 + 2; t.chunk = 0;
     } else {
-        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kPair, kQcPair);
+        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kPair, a.qc);
         t.b = ii.b; t.T = ii.T; t.t0 = ii.t0;
         const int nt = (t.T + kTile - 1) / kTile;
         t.g = ii.g;
         t.kt = 2 * ii.kt;                  // key tiles kt (A) and kt + 1 (B, may be >= nt)
         t.qt0 = 2 * ii.qt0;
         t.qt1 = min(nt, 2 * ii.qt1);
-        t.chunk = (ii.qt0 - ii.kt) / kQcPair;
+        t.chunk = (ii.qt0 - ii.kt) / a.qc;
         t.fix_y = a.hs.group[ii.g];
         t.fix_row0 = t.kt * kTile;
         const int nh = a.hs.begin[ii.g + 1] - a.hs.begin[ii.g];
@@ -712,7 +717,14 @@ estp_status launch_tc(estp_ctx* ctx, const CUtensorMap& fixm, const CUtensorMap&
 
 bool tc_supported(estp_dtype dtype, int d) { return dtype == ESTP_BF16 && (d == 64 || d == 128); }
 int tc_tile() { return kPair; }
-int tc_qc() { return kQcPair; }
+int tc_qc(int B, int64_t sumT, int n_groups, int num_sms) {
+    // the prompts' lengths stay on the device: estimate the item count from the mean length
+    const int64_t t_mean = B > 0 ? (sumT + B - 1) / B : 0;
+    const int64_t nt = (t_mean + kPair - 1) / kPair;
+    for (int qc : kQcChoices)
+        if ((int64_t)B * n_groups * items_f(nt, qc) >= (int64_t)kItemsPerSm * num_sms) return qc;
+    return kQcChoices[3];
+}
 
 estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, int Hkv, int d,
                           float scale, const ImpHeads& hs, const int32_t* cu, int B, int64_t sumT,
@@ -745,9 +757,10 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
 estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const float* lse, int Hq,
                           int Hkv, int d, float scale, const ImpHeads& hs, const int32_t* cu,
                           int B, int64_t sumT, bool exclude_self, const int32_t* base,
-                          const PlanInfo* info, float* part, int c_max, cudaStream_t st) {
+                          const PlanInfo* info, float* part, int c_max, int qc, cudaStream_t st) {
     TcArgs a{};
     a.c_max = c_max;
+    a.qc = qc;
     a.cu = cu; a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.sumT = sumT;
     a.base = base; a.info = info;
     a.scale_log2 = scale * kLog2e;

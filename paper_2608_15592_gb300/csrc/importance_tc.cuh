@@ -6,7 +6,9 @@ namespace estp {
 
 bool tc_supported(estp_dtype dtype, int d);
 int tc_tile();  // keys (and queries) per tile
-int tc_qc();    // query tiles per importance item
+// pairs of query tiles per column-sum item for a call over B prompts, sumT tokens and
+// n_groups KV groups on num_sms SMs
+int tc_qc(int B, int64_t sumT, int n_groups, int num_sms);
 
 estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, int Hkv, int d,
                           float scale, const ImpHeads& hs, const int32_t* cu, int B, int64_t sumT,
@@ -15,6 +17,6 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
 estp_status launch_imp_tc(estp_ctx* ctx, const void* Q, const void* K, const float* lse, int Hq,
                           int Hkv, int d, float scale, const ImpHeads& hs, const int32_t* cu,
                           int B, int64_t sumT, bool exclude_self, const int32_t* base,
-                          const PlanInfo* info, float* part, int c_max, cudaStream_t st);
+                          const PlanInfo* info, float* part, int c_max, int qc, cudaStream_t st);
 
 }  // namespace estp

@@ -213,3 +213,34 @@ def test_importance_workload(cuda_lib, w):
     for b in range(w.B):
         assert abs(S[cu[b]:cu[b + 1]].sum() - 1.0) < 1e-4
     assert_importance(S, oracle.importance(C, cu, len(w.layers), w.Hq))
+
+
+@pytest.mark.parametrize("B,T,expect_qc", [(32, 2048, 4), (16, 4096, 8), (20, 4096, 16)])
+def test_importance_chunk_sizes(cuda_lib, B, T, expect_qc):
+    """Batches large enough that the column-sum items cover 4, 8 and 16 query-tile pairs
+    (the host picks the largest that keeps ~16 items per SM): one head per KV group, every
+    prompt against the oracle element by element."""
+    w = W.Workload("chunks", seed=41 + B, B=B, T_lo=T, T_hi=T, dtype=synth.BF16, V=8,
+                   n_layers_model=1, layers_used=1, Hq=32, Hkv=8, d=128, D=64, sinks=4)
+    # the host's choice, restated: largest qc with B * groups * items(nt, qc) >= 16 * SMs
+    def items_f(n, qc):
+        a, r = n // qc, n % qc
+        return qc * a * (a + 1) // 2 + r * (a + 1)
+    n_sms = torch.cuda.get_device_properties(0).multi_processor_count
+    nt = (T + 255) // 256
+    picked = next((qc for qc in (16, 8, 4, 2) if B * w.Hkv * items_f(nt, qc) >= 16 * n_sms), 2)
+    if picked != expect_qc:
+        pytest.skip(f"{n_sms} SMs pick {picked} query-tile pairs per item, not {expect_qc}")
+    cu = w.cu_seqlens()
+    sumT = int(cu[-1])
+    heads = list(range(0, w.Hq, w.Hq // w.Hkv))  # one per KV group
+    ctx = cuda_lib.Context(0)
+    Q, K = sd.qk(w, w.layers[0])
+    ctx.attn_importance(Q, K, sd.cu_seqlens(w), T, heads=heads)
+    S = ctx.attn_importance_finalize(1, sumT).cpu().numpy()
+    ctx.sync_status()
+    Qh = Q.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    Kh = K.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    C = oracle.attn_colsum(Qh, Kh, cu, w.scale, heads=heads)
+    assert_importance(S, oracle.importance(C, cu, 1, len(heads)))
+    ctx.close()
