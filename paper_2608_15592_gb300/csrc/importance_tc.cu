@@ -24,9 +24,10 @@
 // and with a single issuer the pipe idles through its two waits and commits per step;
 // with one issuer per tile those waits overlap the other tile's MMAs.
 //
-// LSE mode (rows = queries): pair p = query tiles 2p, 2p+1 of one head, streaming the
-//   key tiles 0..2p+1 with a running max (flash-style normaliser); a tile skips the
-//   key tiles after its own query tile.
+// LSE mode (rows = queries): a pair = query tiles q, q+1 of one head (q odd when the
+//   prompt's tile count is odd, so that the unpaired tile is tile 0), streaming the key
+//   tiles 0..q+1 with a running max (flash-style normaliser); a tile skips the key tiles
+//   after its own query tile.
 // Column-sum mode (rows = keys): pair p = key tiles 2p, 2p+1 of one KV group,
 //   C_j += sum_{i>=j} 2^(scale*log2e q_i.k_j - log2e*lse_i), streaming the query tiles
 //   of the item's chunk for every selected head of the group, so the sum over queries
@@ -130,9 +131,12 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
         t.h = a.hs.head_list[li.hslot];
         t.fix_y = t.h;
         const int nt = (t.T + kTile - 1) / kTile;
-        t.qt0 = 2 * li.qt;                 // query tiles qt0 (A) and qt0 + 1 (B, may be >= nt)
-        t.fix_row0 = t.qt0 * kTile;
-        t.n_steps = min(t.qt0 + 2, nt);    // key tiles 0 .. the pair's last tile
+        // Query tiles qt0 (A) and qt0 + 1 (B).  Pairs end at the prompt's last tile, so with
+        // an odd tile count the unpaired tile is tile 0: the pair (-1, 0) streams one key
+        // tile, where a lone last tile would stream all of them for nothing.
+        t.qt0 = 2 * li.qt - (nt & 1);
+        t.fix_row0 = t.qt0 * kTile;        // -128 for that pair: rows outside the prompt
+        t.n_steps = t.qt0 + 2;             // key tiles 0 .. the pair's last tile
         t.g = 0; t.kt = 0; t.qt1 = t.qt0 + 2; t.chunk = 0;
     } else {
         const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kPair, a.qc);
@@ -640,7 +644,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float mm = fmaxf(m, o.x);
                     const float ss = ssum * ex2(m - mm) + o.y * ex2(o.x - mm);
                     const int i = t.fix_row0 + tau * kTile + row;
-                    if (i < t.T && in_bounds(t.h >= 0 && t.h < a.Hq && t.t0 + i < a.sumT, a.status))
+                    if (i >= 0 && i < t.T && in_bounds(t.h >= 0 && t.h < a.Hq && t.t0 + i < a.sumT, a.status))
                         a.lse_out[(int64_t)t.h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
                 }
             }
