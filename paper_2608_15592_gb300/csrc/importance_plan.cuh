@@ -56,10 +56,11 @@ struct ImpItem {
     int T;
 };
 
-__device__ __forceinline__ ImpItem decode_imp_item(int item, const int32_t* base, int B,
-                                                   const int32_t* cu, int tile, int qc) {
+// Item `item` of prompt b (the prompt whose items contain it: upper_slot(base, B, item)).
+__device__ __forceinline__ ImpItem decode_imp_item_at(int item, int b, const int32_t* base,
+                                                      const int32_t* cu, int tile, int qc) {
     ImpItem it;
-    it.b = upper_slot(base, B, item);
+    it.b = b;
     it.t0 = cu[it.b];
     it.T = cu[it.b + 1] - cu[it.b];
     const int nt = (it.T + tile - 1) / tile;
@@ -80,16 +81,21 @@ __device__ __forceinline__ ImpItem decode_imp_item(int item, const int32_t* base
     return it;
 }
 
+__device__ __forceinline__ ImpItem decode_imp_item(int item, const int32_t* base, int B,
+                                                   const int32_t* cu, int tile, int qc) {
+    return decode_imp_item_at(item, upper_slot(base, B, item), base, cu, tile, qc);
+}
+
 struct LseItem {
     int b, hslot, qt;
     int64_t t0;
     int T;
 };
 
-__device__ __forceinline__ LseItem decode_lse_item(int item, const int32_t* base, int B,
-                                                   const int32_t* cu, int tile, int n_heads) {
+__device__ __forceinline__ LseItem decode_lse_item_at(int item, int b, const int32_t* base,
+                                                      const int32_t* cu, int tile, int n_heads) {
     LseItem it;
-    it.b = upper_slot(base, B, item);
+    it.b = b;
     it.t0 = cu[it.b];
     it.T = cu[it.b + 1] - cu[it.b];
     const int nt = (it.T + tile - 1) / tile;
@@ -98,6 +104,11 @@ __device__ __forceinline__ LseItem decode_lse_item(int item, const int32_t* base
     it.hslot = local - rank * n_heads;
     it.qt = nt - 1 - rank;
     return it;
+}
+
+__device__ __forceinline__ LseItem decode_lse_item(int item, const int32_t* base, int B,
+                                                   const int32_t* cu, int tile, int n_heads) {
+    return decode_lse_item_at(item, upper_slot(base, B, item), base, cu, tile, n_heads);
 }
 
 // Number of chunks of key tile kt of a prompt with nt tiles.

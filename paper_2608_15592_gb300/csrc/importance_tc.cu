@@ -85,8 +85,9 @@ struct Cfg {
     // drain[A, B], sched_full/empty[kSched], xfull/xempty[2][A, B][4], lse_full/empty[kLseSlots]
     static constexpr int kNumBars =
         2 + 2 + 2 * kStages + 4 * kAccBufs + 2 + 2 * kSched + 32 + 2 * kLseSlots;
-    static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // tmem addr, abort flag, sched items
-    static constexpr int kLseOff = (kMiscOff + 16 + 4 * kSched + 127) / 128 * 128;  // lse ring
+    // tmem addr, abort flag, then the sched ring's item indices and their prompts (int32)
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;
+    static constexpr int kLseOff = (kMiscOff + 16 + 8 * kSched + 127) / 128 * 128;  // lse ring
     static constexpr int kSmemBytes = kLseOff + kLseSlots * kLseSlotBytes + 1024;  // + alignment slack
 };
 
@@ -122,11 +123,12 @@ struct TcItem {
     int h, g, kt, qt0, qt1, chunk;
 };
 
+// Item `item`, which belongs to prompt b (looked up once by the producer).
 template <int MODE>
-__device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
+__device__ __forceinline__ TcItem make_item(const TcArgs& a, int item, int b) {
     TcItem t;
     if (MODE == kModeLse) {
-        const LseItem li = decode_lse_item(item, a.base, a.B, a.cu, kPair, a.hs.n_heads);
+        const LseItem li = decode_lse_item_at(item, b, a.base, a.cu, kPair, a.hs.n_heads);
         t.b = li.b; t.T = li.T; t.t0 = li.t0;
         t.h = a.hs.head_list[li.hslot];
         t.fix_y = t.h;
@@ -139,7 +141,7 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item) {
         t.n_steps = t.qt0 + 2;             // key tiles 0 .. the pair's last tile
         t.g = 0; t.kt = 0; t.qt1 = t.qt0 + 2; t.chunk = 0;
     } else {
-        const ImpItem ii = decode_imp_item(item, a.base, a.B, a.cu, kPair, a.qc);
+        const ImpItem ii = decode_imp_item_at(item, b, a.base, a.cu, kPair, a.qc);
         t.b = ii.b; t.T = ii.T; t.t0 = ii.t0;
         const int nt = (t.T + kTile - 1) / kTile;
         t.g = ii.g;
@@ -224,6 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::kMiscOff);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 4);
     volatile int* sched_item = reinterpret_cast<volatile int*>(sm + C::kMiscOff + 16);
+    volatile int* sched_b = sched_item + kSched;  // prompt of each published item
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -274,8 +277,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     PlanInfo* info = const_cast<PlanInfo*>(a.info);
     const int total = info->total;
 
-    // Item k of this CTA, published by the producer in slot k % kSched (-1 = no more).
-    auto consume_item = [&](int k, bool warp_uniform) -> int {
+    // Item k of this CTA and its prompt, published by the producer in slot k % kSched
+    // (item -1 = no more).
+    auto consume_item = [&](int k, bool warp_uniform, int& b) -> int {
         const int slot = k % kSched;
         const uint32_t par = (uint32_t)((k / kSched) & 1);
         bool got;
@@ -283,6 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         else got = wait_bar(&sched_full[slot], par, abort_flag, a.status, a.wait_cycles);
         if (!got) return -1;
         const int item = sched_item[slot];
+        b = sched_b[slot];
         if (warp_uniform) __syncwarp();
         if (!warp_uniform || lane == 0) mbar_arrive(&sched_empty[slot]);
         return item;
@@ -307,10 +312,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (it >= kSched &&
                     !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status, a.wait_cycles))
                     break;
+                // the item's prompt: one lookup here instead of one in every consumer role
+                const int b = item >= 0 ? upper_slot(a.base, a.B, item) : 0;
                 sched_item[slot] = item;
-                mbar_arrive(&sched_full[slot]);  // release: the item index is visible to waiters
+                sched_b[slot] = b;
+                mbar_arrive(&sched_full[slot]);  // release: item and prompt visible to waiters
                 if (item < 0) break;
-                const TcItem t = make_item<MODE>(a, item);
+                const TcItem t = make_item<MODE>(a, item, b);
                 const int fb = it & 1;
                 if (it >= 2 && !wait_bar(&fix_empty[fb], ((it >> 1) - 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 mbar_expect_tx(&fix_full[fb], 2 * C::kTileBytes);
@@ -380,9 +388,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t step = 0;
             bool issued = false;
             for (int it = 0;; ++it) {
-                const int item = consume_item(it, false);
+                int b = 0;
+                const int item = consume_item(it, false, b);
                 if (item < 0) break;
-                const TcItem t = make_item<MODE>(a, item);
+                const TcItem t = make_item<MODE>(a, item, b);
                 const int fb = it & 1;
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 const uint32_t fix_addr = smem_u32(fix + (fb * 2 + tau) * C::kTileBytes);
@@ -438,9 +447,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t step = 0;
         bool ok = true;
         for (int it = 0; ok; ++it) {
-            const int item = consume_item(it, true);
+            int b = 0;
+            const int item = consume_item(it, true, b);
             if (item < 0) break;
-            const TcItem t = make_item<MODE>(a, item);
+            const TcItem t = make_item<MODE>(a, item, b);
             // column-sum mode: partial sums of this thread's four key rows 8 s + g8 (s = 0..3)
             // of the quarter, over its columns (16x256b layout, see below)
             float2 acc4[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
