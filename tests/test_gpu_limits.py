@@ -50,7 +50,7 @@ def test_entropy_vocab_extremes(cuda_lib, V):
     ctx.sync_status()
     assert_entropy(H, oracle.token_entropy(_bits(x), V=V))
     if V == 1:
-        assert np.all(H == 0)
+        assert np.max(np.abs(H)) < 1e-6  # a one-entry vocabulary has zero entropy
     ctx.close()
 
 
@@ -69,8 +69,8 @@ def test_many_prompts_and_single_tokens(cuda_lib):
     ctx = cuda_lib.Context(0)
     ctx.attn_importance(Q, K, cu_d, 3)
     S = ctx.attn_importance_finalize(1, sumT).cpu().numpy()
-    x = sd.logits(w, 0, sumT)
-    H = ctx.token_entropy(x, cu_seqlens=cu_d).cpu().numpy()
+    x = sd.logits(w, 0, sumT, ld=304)  # 300 entries in rows of 304 (16-byte stride)
+    H = ctx.token_entropy(x, V=w.V, cu_seqlens=cu_d).cpu().numpy()
     hid = sd.normal(w.key(4), (sumT, w.D), synth.BF16)
     pooled, _ = ctx.pool(hid, torch.as_tensor(H, device="cuda"), torch.as_tensor(S, device="cuda"),
                          cu_d, w.lambda1, w.lambda2, w.alpha)
@@ -79,7 +79,7 @@ def test_many_prompts_and_single_tokens(cuda_lib):
     assert_importance(S, oracle.importance(C, cu, 1, w.Hq))
     one = np.nonzero(lens == 1)[0]
     assert np.all(np.abs(S[cu[one]] - 1.0) < 1e-5)  # a one-token prompt puts all mass on itself
-    assert_entropy(H, oracle.token_entropy(_bits(x)))
+    assert_entropy(H, oracle.token_entropy(_bits(x), V=w.V))
     ref = oracle.pool(_bits(hid), H, S, cu, w.lambda1, w.lambda2, w.alpha)
     P = pooled.cpu().numpy()
     empty = lens == 0
