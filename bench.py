@@ -411,12 +411,11 @@ def run_ours(args, rank, world, local_rank):
 
 # ------------------------------------------------------------- end to end
 class HostPool:
-    """Pinned host copies of the step's inputs for the end-to-end legs, at most
-    HOST_POOL_BYTES in all: the hidden states, Q/K of the first Lp selected layers and
-    the first R rows of the logits (all of them when they fit; the GPU machine has 200 GB of
-    host memory, less than one step's inputs of the RL batch).  A step copies its FULL
-    input size over the host link: layer n's Q/K from pool layer n mod Lp, logit row r
-    from pool row r mod R."""
+    """Pinned host copies of the step's inputs for the end-to-end legs, at most budget()
+    bytes in all: the hidden states, Q/K of the first Lp selected layers and the first R
+    rows of the logits (all of them when they fit; one step of the RL batch needs 315 GB,
+    more than a host may hold).  A step copies its FULL input size over the host link:
+    layer n's Q/K from pool layer n mod Lp, logit row r from pool row r mod R."""
 
     @staticmethod
     def budget() -> int:
