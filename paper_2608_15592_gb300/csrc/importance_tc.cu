@@ -106,6 +106,7 @@ struct TcArgs {
     long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
     int c_max;              // column-sum mode: chunk slots of the partial buffer (bounds checks)
     int qc;                 // column-sum mode: pairs of query tiles per item
+    int head_pairs;         // LSE mode: an item is one query tile of two heads of a group
     ImpHeads hs;
 };
 
@@ -116,11 +117,12 @@ constexpr uint32_t kIdesc = idesc_bf16(kTile, kTile);
 struct TcItem {
     int b, T;
     int64_t t0;
-    int fix_y, fix_row0;       // fixed pair: head (LSE: query head, IMP: KV head), first row
+    int fix_y, fix_row0;       // fixed tile A: head (LSE: query head, IMP: KV head), first row
+    int fix_y2, dq;            // fixed tile B: head, and its tile offset from A (1 or 0)
     int n_steps;
-    // LSE: the query head and the pair's first query tile (qt0);
+    // LSE: the query heads of tiles A and B and tile A's query tile (qt0);
     // IMP: group slot, the pair's first key tile (kt), query-tile range, chunk slot
-    int h, g, kt, qt0, qt1, chunk;
+    int h, h2, g, kt, qt0, qt1, chunk;
 };
 
 // Item `item`, which belongs to prompt b (looked up once by the producer).
@@ -128,18 +130,33 @@ template <int MODE>
 __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item, int b) {
     TcItem t;
     if (MODE == kModeLse) {
-        const LseItem li = decode_lse_item_at(item, b, a.base, a.cu, kPair, a.hs.n_heads);
-        t.b = li.b; t.T = li.T; t.t0 = li.t0;
-        t.h = a.hs.head_list[li.hslot];
+        t.g = 0; t.kt = 0; t.chunk = 0;
+        if (a.head_pairs) {
+            // Query tile qt0 of heads head_list[2u] (A) and head_list[2u + 1] (B), two heads of
+            // one KV group: both need the key tiles 0 .. qt0, so no step leaves a tile idle.
+            const LseItem li = decode_lse_item_at(item, b, a.base, a.cu, kTile, a.hs.n_heads >> 1);
+            t.b = li.b; t.T = li.T; t.t0 = li.t0;
+            t.h = a.hs.head_list[2 * li.hslot];
+            t.h2 = a.hs.head_list[2 * li.hslot + 1];
+            t.qt0 = li.qt;
+            t.dq = 0;
+            t.n_steps = t.qt0 + 1;
+        } else {
+            const LseItem li = decode_lse_item_at(item, b, a.base, a.cu, kPair, a.hs.n_heads);
+            t.b = li.b; t.T = li.T; t.t0 = li.t0;
+            t.h = t.h2 = a.hs.head_list[li.hslot];
+            const int nt = (t.T + kTile - 1) / kTile;
+            // Query tiles qt0 (A) and qt0 + 1 (B).  Pairs end at the prompt's last tile, so
+            // with an odd tile count the unpaired tile is tile 0: the pair (-1, 0) streams one
+            // key tile, where a lone last tile would stream all of them for nothing.
+            t.qt0 = 2 * li.qt - (nt & 1);
+            t.dq = 1;
+            t.n_steps = t.qt0 + 2;         // key tiles 0 .. the pair's last tile
+        }
         t.fix_y = t.h;
-        const int nt = (t.T + kTile - 1) / kTile;
-        // Query tiles qt0 (A) and qt0 + 1 (B).  Pairs end at the prompt's last tile, so with
-        // an odd tile count the unpaired tile is tile 0: the pair (-1, 0) streams one key
-        // tile, where a lone last tile would stream all of them for nothing.
-        t.qt0 = 2 * li.qt - (nt & 1);
-        t.fix_row0 = t.qt0 * kTile;        // -128 for that pair: rows outside the prompt
-        t.n_steps = t.qt0 + 2;             // key tiles 0 .. the pair's last tile
-        t.g = 0; t.kt = 0; t.qt1 = t.qt0 + 2; t.chunk = 0;
+        t.fix_y2 = t.h2;
+        t.fix_row0 = t.qt0 * kTile;        // -128 for the pair (-1, 0): rows outside the prompt
+        t.qt1 = t.qt0 + 1 + t.dq;
     } else {
         const ImpItem ii = decode_imp_item_at(item, b, a.base, a.cu, kPair, a.qc);
         t.b = ii.b; t.T = ii.T; t.t0 = ii.t0;
@@ -149,11 +166,12 @@ __device__ __forceinline__ TcItem make_item(const TcArgs& a, int item, int b) {
         t.qt0 = 2 * ii.qt0;
         t.qt1 = min(nt, 2 * ii.qt1);
         t.chunk = (ii.qt0 - ii.kt) / a.qc;
-        t.fix_y = a.hs.group[ii.g];
+        t.fix_y = t.fix_y2 = a.hs.group[ii.g];
         t.fix_row0 = t.kt * kTile;
+        t.dq = 1;
         const int nh = a.hs.begin[ii.g + 1] - a.hs.begin[ii.g];
         t.n_steps = nh * (t.qt1 - t.qt0);
-        t.h = 0;
+        t.h = t.h2 = 0;
     }
     return t;
 }
@@ -327,7 +345,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int at = 0; at < C::kAtoms; ++at)
                         tma_load_3d(fix + (fb * 2 + tau) * C::kTileBytes + at * kTile * 128, &tm_fix,
-                                    at * 64, t.fix_y, (int)(t.t0 + t.fix_row0) + tau * kTile,
+                                    at * 64, tau ? t.fix_y2 : t.fix_y,
+                                    (int)(t.t0 + t.fix_row0) + tau * t.dq * kTile,
                                     &fix_full[fb]);
                 ++n_items;
                 bool ok = true;
@@ -487,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool imp_skip = MODE == kModeImp && qt < kt;   // queries all before keys
                 const bool imp_diag = MODE == kModeImp && qt == kt;
                 // LSE mode: this warp's query tile against streamed key tile s
-                const int my_qt = t.qt0 + tau;
+                const int my_qt = t.qt0 + tau * t.dq;
                 const bool lse_skip = MODE == kModeLse && s > my_qt;  // keys all after queries
                 const bool lse_diag = MODE == kModeLse && s == my_qt;
                 if (imp_skip || lse_skip) {  // nothing to read: hand the accumulator back
@@ -653,9 +672,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 } else {
                     const float mm = fmaxf(m, o.x);
                     const float ss = ssum * ex2(m - mm) + o.y * ex2(o.x - mm);
-                    const int i = t.fix_row0 + tau * kTile + row;
-                    if (i >= 0 && i < t.T && in_bounds(t.h >= 0 && t.h < a.Hq && t.t0 + i < a.sumT, a.status))
-                        a.lse_out[(int64_t)t.h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
+                    const int i = t.fix_row0 + tau * t.dq * kTile + row;
+                    const int h = tau ? t.h2 : t.h;
+                    if (i >= 0 && i < t.T && in_bounds(h >= 0 && h < a.Hq && t.t0 + i < a.sumT, a.status))
+                        a.lse_out[(int64_t)h * a.sumT + t.t0 + i] = (mm + lg2(ss)) * kLn2;
                 }
             }
         }
@@ -759,8 +779,13 @@ estp_status launch_lse_tc(estp_ctx* ctx, const void* Q, const void* K, int Hq, i
     CUtensorMap mq, mk;
     if ((s = make_map(&mq, Q, Hq, d, sumT)) != ESTP_OK) return s;
     if ((s = make_map(&mk, K, Hkv, d, sumT)) != ESTP_OK) return s;
-    // LSE pair items: (prompt, pair of query tiles, head)
-    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, kPair, 1, hs.n_heads, 1,
+    // LSE items: (prompt, query tile, pair of heads of one KV group) when every group holds
+    // an even number of the selected heads, else (prompt, pair of query tiles, head)
+    a.head_pairs = 1;
+    for (int g = 0; g < hs.n_groups; ++g)
+        if ((hs.begin[g + 1] - hs.begin[g]) & 1) a.head_pairs = 0;
+    attn_plan_kernel<<<1, 1024, 0, st>>>(cu, B, sumT, max_seqlen, a.head_pairs ? kTile : kPair, 1,
+                                         a.head_pairs ? hs.n_heads / 2 : hs.n_heads, 1,
                                          const_cast<int32_t*>(a.base), const_cast<PlanInfo*>(a.info),
                                          ctx->status);
     // (the lse map argument is unused in this mode)
