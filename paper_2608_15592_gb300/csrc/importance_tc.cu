@@ -415,6 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!wait_bar(&fix_full[fb], (it >> 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 const uint32_t fix_addr = smem_u32(fix + (fb * 2 + tau) * C::kTileBytes);
                 bool ok = true;
+                int q_it = t.qt0;  // column sums: the step's query tile
                 for (int s = 0; s < t.n_steps; ++s, ++step) {
                     const int stage = (int)(step % C::kStages);
                     const uint32_t u = step / C::kStages;
@@ -431,14 +432,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_fence_after();
                     issued = true;
+                    // a tile wholly above the diagonal (queries all before keys) is not
+                    // computed: the epilogue skips it, and its commit still hands it over
+                    const bool skip = MODE == kModeImp ? q_it < t.kt + tau : s > t.qt0 + tau * t.dq;
+                    if (!skip) {
 #pragma unroll
-                    for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {  // K steps of 16
-                        const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
-                        mma_bf16<kIdesc>(tmem + (uint32_t)((ab * 2 + tau) * kAccCols), sw128_desc(fix_addr + off),
-                                 sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
+                        for (int kk = 0; kk < 4 * C::kAtoms; ++kk) {  // K steps of 16
+                            const uint32_t off = (uint32_t)((kk >> 2) * kTile * 128 + (kk & 3) * 32);
+                            mma_bf16<kIdesc>(tmem + (uint32_t)((ab * 2 + tau) * kAccCols), sw128_desc(fix_addr + off),
+                                     sw128_desc(str_addr + off), kk > 0 ? 1u : 0u);
+                        }
                     }
                     mma_commit(&acc_full[tau * kAccBufs + ab]);
                     mma_commit(&ring_empty[stage]);
+                    if (MODE == kModeImp && ++q_it == t.qt1) q_it = t.qt0;
                 }
                 if (!ok) break;
                 mma_commit(&fix_empty[fb]);
