@@ -187,16 +187,26 @@ def algorithmic(w, cu):
     }
 
 
+def source_hash(source: str) -> str:
+    """First 16 hex digits of the SHA-256 of a kernel's translation unit followed by every
+    header of the CUDA sources (sorted by name), so that a change to a shared header, too,
+    marks a capture as stale."""
+    csrc = os.path.join(ROOT, "paper_2608_15592_gb300", "csrc")
+    h = hashlib.sha256(open(os.path.join(csrc, source), "rb").read())
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith(".cuh"):
+            h.update(open(os.path.join(csrc, name), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def traffic_for(kernel: str, workload: str):
     """dram bytes per launch from a committed ncu summary, if it was captured for this
-    workload and the kernel's source has not changed since the capture; else None."""
+    workload and the kernel's sources have not changed since the capture; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             t = json.load(f)[workload][kernel]
-        src = os.path.join(ROOT, "paper_2608_15592_gb300", "csrc", t["source"])
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        return t["dram_bytes_per_launch"] if h == t["source_sha256_16"] else None
+        return t["dram_bytes_per_launch"] if source_hash(t["source"]) == t["source_sha256_16"] else None
     except Exception:
         return None
 

@@ -67,3 +67,23 @@ def test_step_launch_count():
     # entropy 2, per layer 2 + 3, finalize 1, pooling 2
     assert bench.lib_launches(W.C4) == 2 + 32 * 5 + 1 + 2
     assert bench.lib_launches(W.C2) == 2 + 4 * 5 + 1 + 2
+
+
+def test_traffic_is_dropped_when_a_kernel_source_or_shared_header_changes(tmp_path, monkeypatch):
+    csrc = tmp_path / "paper_2608_15592_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "profiles").mkdir()
+    (csrc / "k.cu").write_text("kernel\n")
+    (csrc / "h.cuh").write_text("header\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    rec = {"wl": {"k": {"source": "k.cu", "source_sha256_16": bench.source_hash("k.cu"),
+                        "dram_bytes_per_launch": 123}}}
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(rec))
+    assert bench.traffic_for("k", "wl") == 123
+    assert bench.traffic_for("k", "other") is None and bench.traffic_for("x", "wl") is None
+    (csrc / "h.cuh").write_text("header, changed\n")
+    assert bench.traffic_for("k", "wl") is None
+    (csrc / "h.cuh").write_text("header\n")
+    assert bench.traffic_for("k", "wl") == 123
+    (csrc / "k.cu").write_text("kernel, changed\n")
+    assert bench.traffic_for("k", "wl") is None
