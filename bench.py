@@ -163,6 +163,22 @@ def layer_qk_bytes(w, sumT: int) -> int:
     return sumT * (w.Hq + w.Hkv) * w.d * esize(w)
 
 
+def input_bytes(w, sumT: int) -> int:
+    """Bytes of one step's inputs (logits, every selected layer's Q/K, hidden states)."""
+    return sumT * w.V * esize(w) + len(w.layers) * layer_qk_bytes(w, sumT) + sumT * w.D * esize(w)
+
+
+def l2_flush_buffer(w, sumT: int, device):
+    """A buffer of twice the L2 size, written between timed steps when a step's inputs
+    are smaller than that (else None: the inputs themselves push the previous step's
+    lines out of L2)."""
+    import torch
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    if input_bytes(w, sumT) >= 2 * l2:
+        return None
+    return torch.empty(2 * l2, dtype=torch.uint8, device=device)
+
+
 def resident_bytes(w) -> int:
     """Device bytes of the step's inputs and outputs when every layer is resident."""
     sumT = int(w.cu_seqlens()[-1])
@@ -320,6 +336,9 @@ def run_ours(args, rank, world, local_rank):
     K = args.steps
     ev = {name: [] for name in Step.CALLS}
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # small inputs: L2 written over between steps, each step timed on its own
+    flush = None if stream_qk else l2_flush_buffer(w, sumT, dev)
+    marks = []
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -328,14 +347,21 @@ def run_ours(args, rank, world, local_rank):
         t_host0 = time.time()
         start.record()
         for k in range(K):
+            if flush is not None:
+                flush.zero_()
+                marks.append((torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)))
+                marks[-1][0].record()
             st.run(ev)
+            if flush is not None:
+                marks[-1][1].record()
         end.record()
         torch.cuda.synchronize()
         clk.window(t_host0, time.time())
     if world > 1:
         torch.distributed.barrier()
     st.ctx.sync_status()
-    region_ms = start.elapsed_time(end)
+    region_ms = (sum(a.elapsed_time(b) for a, b in marks) if flush is not None
+                 else start.elapsed_time(end))
     call_ms = {name: sum(a.elapsed_time(b) for a, b in ev[name]) for name in Step.CALLS}
     calls_total = sum(call_ms.values())
     # resident inputs: the whole region is library work; streamed Q/K: the calls only
@@ -380,6 +406,8 @@ def run_ours(args, rank, world, local_rank):
         e2e_hidden = run_e2e_from_hidden(args, st, pool, dev, world)
         del pool
     side = {}
+    if not stream_qk:
+        side["graph_replay"] = time_graph(st, K, flush)
     if not args.no_side:
         side["head_loss"] = time_head_loss(st, dev)
         side["misalignment"] = time_misalignment(st)
@@ -395,8 +423,11 @@ def run_ours(args, rank, world, local_rank):
                "parallelism": f"dp{world} (independent prompts)",
                "qk": "generated per layer (streamed)" if stream_qk else "resident",
                "timing": timing,
-               "l2": f"inputs larger than L2 ({(sumT * w.V * esize(w)) / 1e9:.1f} GB of logits "
-                     "per step), no flush"}
+               "l2": (f"inputs larger than L2 ({(sumT * w.V * esize(w)) / 1e9:.1f} GB of logits "
+                      "per step), no flush") if flush is None else
+                     (f"inputs of {input_bytes(w, sumT) / 1e6:.1f} MB, under twice the L2: a "
+                      f"{flush.numel() / 2**20:.0f} MiB buffer written between steps, outside "
+                      "each step's events")}
     gen_per_step = (st.n_layers * (2 + (1 if w.sinks else 0))) if stream_qk else 0
     del st
     if rank != 0:
@@ -672,6 +703,48 @@ def run_e2e_from_hidden(args, st, pool, dev, world):
 
 
 # ------------------------------------------------------- side measurements
+def time_graph(st, K: int, flush):
+    """The same step captured once in a CUDA graph and replayed K times (resident
+    workloads only): the library calls enqueue nothing that a graph cannot hold (no
+    allocation once the workspace has grown, no synchronisation), so a replay launches
+    the step's kernels without the host's per-call work.  Each replay is timed with CUDA
+    events, with the L2 written over in between when the inputs are small.  The outputs of
+    a replay are checked bit for bit against the step run call by call."""
+    import torch
+    st.run()
+    torch.cuda.synchronize()
+    ref = [t.clone() for t in (st.H, st.S, st.pooled, st.pred)]
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        st.run()
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        st.run()
+    for t in (st.H, st.S, st.pooled, st.pred):
+        t.fill_(float("nan"))
+    g.replay()
+    torch.cuda.synchronize()
+    same = all(torch.equal(a, b) for a, b in zip(ref, (st.H, st.S, st.pooled, st.pred)))
+    ms = []
+    for _ in range(K):
+        if flush is not None:
+            flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        g.replay()
+        b.record()
+        ms.append((a, b))
+    torch.cuda.synchronize()
+    st.ctx.sync_status()
+    per = sum(a.elapsed_time(b) for a, b in ms) / K
+    del g
+    return {"ms_per_step": per, "value": st.sumT / (per / 1e3), "unit": UNIT, "steps": K,
+            "launches_per_step": lib_launches(st.w), "bit_equal_to_calls": same}
+
+
+
 def _time_calls(fn, sync, min_warm_s: float = 0.5, want_s: float = 1.5, min_iters: int = 3):
     """CUDA-event time of one fn() after at least min_warm_s (and two calls) of warm-up;
     the number of timed calls targets want_s.  Returns ms per call."""
