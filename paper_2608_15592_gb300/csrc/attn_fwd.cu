@@ -96,6 +96,7 @@ struct FwdArgs {
     float* part;            // [slots][128]
     int64_t n_slots;        // slots of part (bounds checks of debug builds)
     int* status;
+    long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
 };
 
 // O += P V: A from TMEM, B an MN-major shared-memory tile (+ D when acc != 0).
@@ -236,8 +237,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = k % kSched;
         const uint32_t par = (uint32_t)((k / kSched) & 1);
         bool got;
-        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status);
-        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status);
+        if (warp_uniform) got = warp_wait(&sched_full[slot], par, abort_flag, a.status, a.wait_cycles);
+        else got = wait_bar(&sched_full[slot], par, abort_flag, a.status, a.wait_cycles);
         FwdItem t{};
         if (!got) return t;
         t = sched_item[slot];
@@ -264,21 +265,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int stage = (int)(v.step & 1);
                 const uint32_t u = v.step >> 1;
                 // P V of step - 2 is complete (p_empty completes with it): its V slot is free
-                if (u >= 1 && !wait_bar(&p_empty[stage], (u - 1) & 1, abort_flag, a.status)) return false;
+                if (u >= 1 && !wait_bar(&p_empty[stage], (u - 1) & 1, abort_flag, a.status, a.wait_cycles)) return false;
                 mbar_expect_tx(&v_full[stage], kTileBytes);
                 for (int at = 0; at < 2; ++at)
                     tma_load_3d(sm + kVOff + stage * kTileBytes + at * kAtomBytes, &tm_v,
                                 at * 64, v.g, v.pos, &v_full[stage]);
                 return true;
             };
-            uint32_t step = 0, v_issued = 0;
+            // K copies issued (copy n into ring slot n % kKStages): counted apart from the
+            // steps, because a step whose V load gives up leaves the loop after its K copy
+            uint32_t step = 0, v_issued = 0, k_issued = 0;
             int n_items = 0;
             int item = blockIdx.x;
             for (int it = 0; ok; ++it) {
                 if (item >= total) item = -1;
                 const int slot = it % kSched;
                 if (it >= kSched &&
-                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status))
+                    !wait_bar(&sched_empty[slot], (uint32_t)(((it / kSched) - 1) & 1), abort_flag, a.status, a.wait_cycles))
                     break;
                 FwdItem t{};
                 if (item >= 0) t = fwd_item(a, item);
@@ -287,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (item < 0) break;
                 const int g = t.h / (a.Hq / a.Hkv);
                 const int fb = it % kQBufs;
-                if (it >= kQBufs && !wait_bar(&q_empty[fb], ((it / kQBufs) - 1) & 1, abort_flag, a.status)) break;
+                if (it >= kQBufs && !wait_bar(&q_empty[fb], ((it / kQBufs) - 1) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 mbar_expect_tx(&q_full[fb], kTileBytes);
                 for (int at = 0; at < 2; ++at)
                     tma_load_3d(sm + kQOff + fb * kTileBytes + at * kAtomBytes, &tm_q, at * 64, t.h,
@@ -296,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int stage = (int)(step % kKStages);
                     const uint32_t u = step / kKStages;
-                    if (u >= 1 && !wait_bar(&k_empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                    if (u >= 1 && !wait_bar(&k_empty[stage], (u - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                         ok = false;
                         break;
                     }
@@ -304,6 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int at = 0; at < 2; ++at)
                         tma_load_3d(sm + kKOff + stage * kTileBytes + at * kAtomBytes, &tm_k, at * 64, g,
                                     (int)(t.t0 + kt * kT), &k_full[stage]);
+                    ++k_issued;
                     if (have_v) {
                         if (!load_v(vp)) {
                             ok = false;
@@ -319,8 +323,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (ok && have_v && load_v(vp)) ++v_issued;
             // every copy in flight lands before the CTA exits
-            for (uint32_t i = 0; i < (uint32_t)kKStages && i < step; ++i)
-                drain_wait(&k_full[(step - 1 - i) % kKStages], ((step - 1 - i) / kKStages) & 1, a.status);
+            for (uint32_t i = 0; i < (uint32_t)kKStages && i < k_issued; ++i)
+                drain_wait(&k_full[(k_issued - 1 - i) % kKStages], ((k_issued - 1 - i) / kKStages) & 1,
+                           a.status);
             for (uint32_t i = 0; i < 2 && i < v_issued; ++i)
                 drain_wait(&v_full[(v_issued - 1 - i) & 1], ((v_issued - 1 - i) >> 1) & 1, a.status);
             for (int i = 0; i < kQBufs && i < n_items; ++i) {  // the last load of each Q buffer
@@ -337,14 +342,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const FwdItem t = consume_item(it, false);
                 if (!t.valid) break;
                 const int fb = it % kQBufs;
-                if (!wait_bar(&q_full[fb], (it / kQBufs) & 1, abort_flag, a.status)) break;
+                if (!wait_bar(&q_full[fb], (it / kQBufs) & 1, abort_flag, a.status, a.wait_cycles)) break;
                 const uint32_t qa = smem_u32(sm + kQOff + fb * kTileBytes);
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int kst = (int)(step % kKStages);
                     const int stage = (int)(step & 1);  // S buffer
                     const uint32_t u = step >> 1;
-                    if (!wait_bar(&k_full[kst], (step / kKStages) & 1, abort_flag, a.status) ||
-                        (u >= 1 && !wait_bar(&s_empty[stage], (u - 1) & 1, abort_flag, a.status))) {
+                    if (!wait_bar(&k_full[kst], (step / kKStages) & 1, abort_flag, a.status, a.wait_cycles) ||
+                        (u >= 1 && !wait_bar(&s_empty[stage], (u - 1) & 1, abort_flag, a.status, a.wait_cycles))) {
                         ok = false;
                         break;
                     }
@@ -380,9 +385,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!t.valid) break;
                 for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                     const int pb = (int)(step & 1);
-                    if (!wait_bar(&v_full[pb], (step >> 1) & 1, abort_flag, a.status) ||
-                        !wait_bar(&p_full[pb], (step >> 1) & 1, abort_flag, a.status) ||
-                        (kt == 0 && it >= 1 && !wait_bar(o_empty, (it - 1) & 1, abort_flag, a.status))) {
+                    if (!wait_bar(&v_full[pb], (step >> 1) & 1, abort_flag, a.status, a.wait_cycles) ||
+                        !wait_bar(&p_full[pb], (step >> 1) & 1, abort_flag, a.status, a.wait_cycles) ||
+                        (kt == 0 && it >= 1 && !wait_bar(o_empty, (it - 1) & 1, abort_flag, a.status, a.wait_cycles))) {
                         ok = false;
                         break;
                     }
@@ -414,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!t.valid) break;
             for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                 const int sb = (int)(step & 1);
-                if (!warp_wait(&cs_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
+                if (!warp_wait(&cs_full[sb], (step >> 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                     ok = false;
                     break;
                 }
@@ -457,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kt = 0; kt <= t.qt; ++kt, ++step) {
                 if ((int)(step & 1) != grp) continue;
                 const int sb = grp;
-                if (!warp_wait(&s_full[sb], (step >> 1) & 1, abort_flag, a.status)) {
+                if (!warp_wait(&s_full[sb], (step >> 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                     ok = false;
                     break;
                 }
@@ -517,13 +522,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 // the reducer warp is done with this buffer's sums of step - 2
-                if (step >= 2 && !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                if (step >= 2 && !warp_wait(&cs_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                     ok = false;
                     break;
                 }
                 *reinterpret_cast<float2*>(csb + q * kT + half * 64 + 2 * lane) = make_float2(csum[0], csum[1]);
                 // P V of step - 2 has read this P buffer
-                if (step >= 2 && !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status)) {
+                if (step >= 2 && !warp_wait(&p_empty[sb], ((step >> 1) - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                     ok = false;
                     break;
                 }
@@ -540,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
             if ((int)((step - 1) & 1) != grp) continue;  // the other group ends this item
             // O of the item: this warp's 32 rows x 64 columns
-            if (!warp_wait(&o_full[grp], n_out & 1, abort_flag, a.status)) break;
+            if (!warp_wait(&o_full[grp], n_out & 1, abort_flag, a.status, a.wait_cycles)) break;
             ++n_out;
             tc_fence_after();
 #pragma unroll
@@ -701,6 +706,7 @@ estp_status launch_attn_forward(estp_ctx* ctx, const void* Q, const void* K, con
     a.exclude_self = exclude_self ? 1 : 0;
     a.lse = lse; a.O = static_cast<__nv_bfloat16*>(O); a.part = part; a.status = ctx->status;
     a.n_slots = slots_bound;
+    a.wait_cycles = ctx->wait_cycles;
     e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return cuda_fail(e, "attention forward smem attribute");
     cudaLaunchConfig_t cf = config(dim3((unsigned)ctx->num_sms), dim3(kThreads), kSmemBytes);

@@ -1,12 +1,14 @@
 """Failure detection on the GPU: a bounded wait that runs out (no fault, no hang).
 
 estp_set_wait_limit lowers the limit of the tensor-core attention kernels' abortable
-waits to a few cycles, far below the latency of a tile copy, so they expire in every
-CTA.  The call must then report ESTP_ERR_TIMEOUT through estp_sync_status (the kernels
-drain the copies and MMAs they issued and free their tensor memory), and the next
-normal call on the same context must match the oracle."""
+waits (row normalisers, column sums, the fused prefill forward) to a few cycles, far
+below the latency of a tile copy, so they expire in every CTA.  The call must then
+report ESTP_ERR_TIMEOUT through estp_sync_status (the kernels drain the copies and MMAs
+they issued and free their tensor memory), and the next normal call on the same
+context must match the oracle."""
 import numpy as np
 import pytest
+import torch
 
 import oracle
 import synth
@@ -48,6 +50,42 @@ def test_wait_runs_out_then_context_recovers(cuda_lib, lse_given):
     S = ctx.attn_importance_finalize(1, sumT).cpu().numpy()
     ctx.sync_status()
     assert_importance(S, _oracle_S(w))
+    ctx.close()
+
+
+@pytest.mark.parametrize("lse_given", [False, True], ids=["lse_computed", "lse_given"])
+def test_forward_wait_runs_out_then_context_recovers(cuda_lib, lse_given):
+    """The same for the fused prefill forward (O = A V with the column sums): its waits
+    run out, the call reports ESTP_ERR_TIMEOUT, and the next call matches the oracle in
+    both O and the importance."""
+    w = WL
+    cu = w.cu_seqlens()
+    sumT, maxT = int(cu[-1]), int(np.diff(cu).max())
+    layer = w.layers[0]
+    Q, K = sd.qk(w, layer)
+    Vh = synth.round_to(synth.normal(w.key_v(layer), np.arange(sumT * w.Hkv * w.d)),
+                        w.dtype).reshape(sumT, w.Hkv, w.d)
+    V = torch.from_numpy(Vh.view(np.int16)).view(torch.bfloat16).cuda()
+    cu_d = sd.cu_seqlens(w)
+    ctx = cuda_lib.Context(0)
+    lse = ctx.attn_lse(Q, K, cu_d, maxT) if lse_given else None
+    ctx.sync_status()
+    ctx.set_wait_limit(2)
+    ctx.attn_forward_importance(Q, K, V, cu_d, maxT, lse=lse)
+    with pytest.raises(cuda_lib.EstpError) as err:
+        ctx.sync_status()
+    assert err.value.status == cuda_lib.ESTP_ERR_TIMEOUT
+    ctx.sync_status()
+    ctx.set_wait_limit(0)
+    O = ctx.attn_forward_importance(Q, K, V, cu_d, maxT, lse=lse)
+    S = ctx.attn_importance_finalize(1, sumT).cpu().numpy()
+    ctx.sync_status()
+    assert_importance(S, _oracle_S(w))
+    Qh, Kh = W.host_qk(w, layer)
+    O_ref = oracle.attn_output(Qh, Kh, Vh, cu, w.scale)
+    vmax = float(np.max(np.abs(synth.bf16_bits_to_f32(Vh))))
+    err = float(np.max(np.abs(O.float().cpu().numpy() - O_ref)))
+    assert err <= 5e-3 * vmax, f"O max abs err {err:.3e}"
     ctx.close()
 
 
