@@ -77,8 +77,9 @@ estp_status estp_sync_status(estp_ctx* ctx, estp_stream_t stream);
 /* Testing aid for the failure path; the paper has no counterpart.  Sets, for this
  * context's later calls, the limit in SM clock cycles of the abortable waits of the
  * tensor-core attention kernels (the row normalisers and column sums of
- * estp_attn_lse / estp_attn_importance on bf16 inputs, and the fused prefill forward of
- * estp_attn_forward_importance).  cycles <= 0 restores the
+ * estp_attn_lse / estp_attn_importance on bf16 inputs, the fused prefill forward of
+ * estp_attn_forward_importance) and of the output-projection kernel of
+ * estp_lm_head_entropy.  cycles <= 0 restores the
  * default, about 2 s.  A limit far below a tile copy's latency makes those waits
  * expire: each CTA then records ESTP_ERR_TIMEOUT in the status word, skips the rest of
  * its work, and waits (with the full default limit) for the copies and MMAs it has

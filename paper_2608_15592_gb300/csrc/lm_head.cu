@@ -21,7 +21,8 @@
 //   M = max m_k, S = sum 2^(m_k - M) s_k, T = sum 2^(m_k - M) (t_k + s_k (m_k - M)),
 // and writes H = ln 2 (log2 S - T / S) (nats).
 //
-// Every mbarrier wait is bounded; on expiry the CTA records ESTP_ERR_TIMEOUT in the status
+// Every mbarrier wait is bounded (a test may lower the limit of the abortable waits
+// through estp_set_wait_limit); on expiry the CTA records ESTP_ERR_TIMEOUT in the status
 // word, drains its own copies and MMAs and frees its TMEM.
 #include "tcgen05.cuh"
 
@@ -58,6 +59,7 @@ struct LmArgs {
     int64_t n_items;   // row blocks x splits
     float* part;       // [3][S][n_rows]: m, s, t (log2 units)
     int* status;
+    long long wait_cycles;  // limit of the abortable waits (kWaitCycles unless a test lowers it)
 };
 
 // Vocabulary tiles [vt0, vt1) of split sp.
@@ -163,7 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int kc = 0; kc < a.nk; ++kc, ++step) {
                         const int stage = (int)(step % kStages);
                         const uint32_t u = step / kStages;
-                        if (u >= 1 && !wait_bar(&empty[stage], (u - 1) & 1, abort_flag, a.status)) {
+                        if (u >= 1 && !wait_bar(&empty[stage], (u - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                             ok = false;
                             break;
                         }
@@ -190,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int vt = vt0; ok && vt < vt1; ++vt, ++tile) {
                     const int ab = (int)(tile % kAccBufs);
                     const uint32_t ua = tile / kAccBufs;
-                    if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status)) {
+                    if (ua >= 1 && !wait_bar(&acc_empty[ab], (ua - 1) & 1, abort_flag, a.status, a.wait_cycles)) {
                         ok = false;
                         break;
                     }
@@ -198,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t d = tmem + (uint32_t)(ab * kN);
                     for (int kc = 0; kc < a.nk; ++kc, ++step) {
                         const int stage = (int)(step % kStages);
-                        if (!wait_bar(&full[stage], (step / kStages) & 1, abort_flag, a.status)) {
+                        if (!wait_bar(&full[stage], (step / kStages) & 1, abort_flag, a.status, a.wait_cycles)) {
                             ok = false;
                             break;
                         }
@@ -232,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float m = -INFINITY, s = 0.f, t = 0.f;
             for (int vt = vt0; vt < vt1; ++vt, ++tile) {
                 const int ab = (int)(tile % kAccBufs);
-                if (!warp_wait(&acc_full[ab], (tile / kAccBufs) & 1, abort_flag, a.status)) {
+                if (!warp_wait(&acc_full[ab], (tile / kAccBufs) & 1, abort_flag, a.status, a.wait_cycles)) {
                     ok = false;
                     break;
                 }
@@ -358,6 +360,7 @@ estp_status launch_lm_head_entropy(estp_ctx* ctx, const void* hidden, int64_t ld
     if (s != ESTP_OK) return s;
     a.part = static_cast<float*>(ctx->ws);
     a.status = ctx->status;
+    a.wait_cycles = ctx->wait_cycles;
     cudaError_t e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kSmemBytes);
     if (e != cudaSuccess) return cuda_fail(e, "lm-head kernel smem attribute");

@@ -1,11 +1,11 @@
 """Failure detection on the GPU: a bounded wait that runs out (no fault, no hang).
 
-estp_set_wait_limit lowers the limit of the tensor-core attention kernels' abortable
-waits (row normalisers, column sums, the fused prefill forward) to a few cycles, far
-below the latency of a tile copy, so they expire in every CTA.  The call must then
-report ESTP_ERR_TIMEOUT through estp_sync_status (the kernels drain the copies and MMAs
-they issued and free their tensor memory), and the next normal call on the same
-context must match the oracle."""
+estp_set_wait_limit lowers the limit of the tensor-core kernels' abortable waits (row
+normalisers, column sums, the fused prefill forward, the entropy from hidden states) to
+a few cycles, far below the latency of a tile copy, so they expire in every CTA.  The
+call must then report ESTP_ERR_TIMEOUT through estp_sync_status (the kernels drain the
+copies and MMAs they issued and free their tensor memory), and the next normal call on
+the same context must match the oracle."""
 import numpy as np
 import pytest
 import torch
@@ -86,6 +86,28 @@ def test_forward_wait_runs_out_then_context_recovers(cuda_lib, lse_given):
     vmax = float(np.max(np.abs(synth.bf16_bits_to_f32(Vh))))
     err = float(np.max(np.abs(O.float().cpu().numpy() - O_ref)))
     assert err <= 5e-3 * vmax, f"O max abs err {err:.3e}"
+    ctx.close()
+
+
+def test_lm_head_wait_runs_out_then_context_recovers(cuda_lib):
+    """The same for the entropy with the logits formed from hidden states: its waits run
+    out, the call reports ESTP_ERR_TIMEOUT, and the next call matches the oracle."""
+    rows, D, V = 300, 192, 1000
+    h = sd.normal(synth.stream_key(23, 7), (rows, D), synth.BF16)
+    Wo = sd.normal(synth.stream_key(23, 8), (V, D), synth.BF16, scale=3.0 / np.sqrt(D))
+    ctx = cuda_lib.Context(0)
+    ctx.set_wait_limit(2)
+    ctx.lm_head_entropy(h, Wo)
+    with pytest.raises(cuda_lib.EstpError) as err:
+        ctx.sync_status()
+    assert err.value.status == cuda_lib.ESTP_ERR_TIMEOUT
+    ctx.sync_status()
+    ctx.set_wait_limit(0)
+    H = ctx.lm_head_entropy(h, Wo).cpu().numpy()
+    ctx.sync_status()
+    bits = lambda t: t.view(torch.int16).cpu().numpy().view(np.uint16)
+    ref = oracle.lm_head_entropy(bits(h), bits(Wo))
+    assert np.max(np.abs(H - ref)) <= 1e-3
     ctx.close()
 
 
