@@ -429,15 +429,20 @@ def run_ours(args, rank, world, local_rank):
                       f"{flush.numel() / 2**20:.0f} MiB buffer written between steps, outside "
                       "each step's events")}
     gen_per_step = (st.n_layers * (2 + (1 if w.sinks else 0))) if stream_qk else 0
+    sample = gpu_sample = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = OracleSample(w)
+        gpu_sample = sample.gpu_outputs(st)
     del st
     if rank != 0:
         return None
-    cpu = None if (world > 1 or args.no_cpu_baseline) else cpu_baseline(w)
+    cpu, parity = cpu_baseline(sample, gpu_sample) if sample is not None else (None, None)
     res = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": out_cfg, "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu,
+        "parity": parity,
         "e2e": e2e, "gpu_launches": lib_launches(w) * K, "clocks": clocks,
         "region_ms_per_step": region_ms / K, "calls_ms_per_step": calls_total / K,
         # context: a prefill's flash attention returns the row normalisers, and the path
@@ -970,6 +975,8 @@ class OracleSample:
                           / (pairs * len(self.heads)))
         self.ratio_pool = self.sumT / Tp
         rows_txt = "all rows" if r0 == 0 else f"query rows {r0}..{T - 1}"
+        self.b, self.T = b, T
+        self.H = self.C = None
         self.desc = (f"entropy {len(self.ent_rows)} rows; importance: the {T}-token prompt "
                      f"(nearest the median), {rows_txt}, 1 layer x {len(self.heads)} of {w.Hq} "
                      f"heads; pooling + head on its first {min(T, 4096)} tokens; extrapolated by algorithmic work "
@@ -993,19 +1000,56 @@ class OracleSample:
                         w.lambda2, w.alpha)
         oracle.length_head(P, *self.head)
         t3 = time.perf_counter()
+        self.H, self.C = H, C
         batch = ((t1 - t0) * self.ratio_ent + (t2 - t1) * self.ratio_imp
                  + (t3 - t2) * self.ratio_pool)
         return t3 - t0, batch
 
 
-def cpu_baseline(w, repeats: int = 3):
-    s = OracleSample(w)
+    def gpu_outputs(self, st):
+        """The library's results on the sample, for the parity record: the step's entropy
+        of the sampled rows, and the importance of the sampled prompt alone (its rows of
+        the last selected layer's Q and K, the sample's heads, one layer, lse computed by
+        the call)."""
+        import torch
+        w = self.w
+        H = st.H[torch.as_tensor(self.ent_rows, device=st.H.device)].cpu().numpy()
+        Q, K = st.qk(len(w.layers) - 1)
+        r0, r1 = int(self.rows[0]), int(self.rows[-1]) + 1
+        cu = torch.as_tensor([0, self.T], dtype=torch.int32, device=Q.device)
+        st.ctx.attn_importance(Q[r0:r1], K[r0:r1], cu, self.T, heads=[int(h) for h in self.heads])
+        S = st.ctx.attn_importance_finalize(1, self.T).cpu().numpy()
+        st.ctx.sync_status()
+        return H, S
+
+    def parity(self, gpu):
+        """Largest errors of the library against the oracle on the sample: entropy (nats,
+        absolute) on the sampled rows; importance (relative, element by element) on the keys
+        the sample's query rows fix exactly (every key when the sample holds all rows)."""
+        import numpy as np
+        H_gpu, S_gpu = gpu
+        S_ref = self.C / (self.T * len(self.heads))
+        keys = np.arange(self.row_from, self.T)
+        rel = np.abs(S_gpu[keys] - S_ref[keys]) / np.maximum(np.abs(S_ref[keys]), 1e-30)
+        return {"entropy_max_abs_err_nats": float(np.max(np.abs(H_gpu - self.H))),
+                "entropy_rows": int(len(self.ent_rows)),
+                "importance_max_rel_err": float(rel.max()) if rel.size else 0.0,
+                "importance_keys": int(len(keys)),
+                "importance_sample": f"prompt {self.b} ({self.T} tokens), last selected layer, "
+                                     f"{len(self.heads)} of {self.w.Hq} heads",
+                "tolerance": {"entropy_nats": 1e-3, "importance_rel": 1e-2}}
+
+
+def cpu_baseline(s, gpu=None, repeats: int = 3):
+    """The oracle timed on the sample s (median of `repeats` passes), and, with the
+    library's outputs on the same sample (OracleSample.gpu_outputs), the parity record."""
     runs = [s.run() for _ in range(repeats)]
     batch = statistics.median(r[1] for r in runs)
-    return {"value": s.sumT / batch, "unit": UNIT, "cores": s.n_threads, "kind": "oracle",
-            "sample": s.desc + f"; median of {repeats} passes of "
-                               f"{statistics.median(r[0] for r in runs):.1f} s",
-            "extrapolated": True}
+    cpu = {"value": s.sumT / batch, "unit": UNIT, "cores": s.n_threads, "kind": "oracle",
+           "sample": s.desc + f"; median of {repeats} passes of "
+                              f"{statistics.median(r[0] for r in runs):.1f} s",
+           "extrapolated": True}
+    return cpu, (s.parity(gpu) if gpu is not None else None)
 
 
 def run_reference(args, rank, world):

@@ -24,6 +24,25 @@ def test_oracle_sample_ratios_cover_the_batch():
     assert wall > 0 and abs(batch - wall) <= 0.5 * wall + 1e-3
 
 
+def test_parity_record_of_the_sample():
+    # outputs equal to the oracle's give zero errors; a planted error in one sampled row
+    # and one key shows up in the record with its size
+    w = W.Workload("tiny", seed=6, B=2, T_lo=20, T_hi=40, dtype="bf16", V=50,
+                   n_layers_model=1, layers_used=1, Hq=4, Hkv=2, d=64, D=32)
+    s = bench.OracleSample(w)
+    s.run()
+    S = s.C / (s.T * len(s.heads))
+    p = s.parity((s.H.copy(), S.copy()))
+    assert p["entropy_max_abs_err_nats"] == 0.0 and p["importance_max_rel_err"] == 0.0
+    assert p["importance_keys"] == s.T and p["entropy_rows"] == len(s.ent_rows)
+    H_bad, S_bad = s.H.copy(), S.copy()
+    H_bad[3] += 2e-3
+    S_bad[s.T - 1] *= 1.05
+    p = s.parity((H_bad, S_bad))
+    assert abs(p["entropy_max_abs_err_nats"] - 2e-3) < 1e-9
+    assert abs(p["importance_max_rel_err"] - 0.05) < 1e-6
+
+
 def test_oracle_sample_long_prompt_uses_last_rows():
     # a 32768-token prompt exceeds the pair budget: one head per thread (8 here), its last
     # query rows only, the first row the one that keeps the pairs within budget
