@@ -215,16 +215,23 @@ def source_hash(source: str) -> str:
     return h.hexdigest()[:16]
 
 
-def traffic_for(kernel: str, workload: str):
-    """dram bytes per launch from a committed ncu summary, if it was captured for this
-    workload and the kernel's sources have not changed since the capture; else None."""
+def counters_for(kernel: str, workload: str):
+    """The committed ncu record of a kernel (profiles/traffic.json: dram bytes per launch,
+    and for the tensor-core kernels the tensor pipe's active share), if it was captured for
+    this workload and the kernel's sources have not changed since the capture; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             t = json.load(f)[workload][kernel]
-        return t["dram_bytes_per_launch"] if source_hash(t["source"]) == t["source_sha256_16"] else None
+        return t if source_hash(t["source"]) == t["source_sha256_16"] else None
     except Exception:
         return None
+
+
+def traffic_for(kernel: str, workload: str):
+    """dram bytes per launch from the committed ncu record (counters_for), else None."""
+    t = counters_for(kernel, workload)
+    return t["dram_bytes_per_launch"] if t else None
 
 
 def lib_launches(w) -> int:
@@ -397,6 +404,14 @@ def run_ours(args, rank, world, local_rank):
                 "frac": dk["frac"], "traffic": traffic_for(dom, w.name),
                 "peak_source": f"{peak_src} ({'hbm_gbs' if dk['bound'] == 'hbm' else 'bf16_tflops_sustained'})",
                 "share_of_step": share[dom] / sum(share.values())}
+    for name, rec in kernels.items():  # the committed ncu counters that still apply
+        c = counters_for(name, w.name)
+        if c:
+            rec["ncu"] = {"dram_bytes_per_launch": c["dram_bytes_per_launch"]}
+            if "tensor_pipe_active_pct" in c:
+                rec["ncu"]["tensor_pipe_active_pct"] = c["tensor_pipe_active_pct"]
+    if dk["bound"] == "tensor" and "ncu" in dk and "tensor_pipe_active_pct" in dk["ncu"]:
+        roofline["tensor_pipe_active_pct"] = dk["ncu"]["tensor_pipe_active_pct"]
     clocks = clk.summary()
 
     e2e = e2e_hidden = None
