@@ -414,6 +414,14 @@ def run_ours(args, rank, world, local_rank):
         roofline["tensor_pipe_active_pct"] = dk["ncu"]["tensor_pipe_active_pct"]
     clocks = clk.summary()
 
+    # the library's outputs on the oracle's sample, taken while the step's inputs and
+    # outputs are still those of the timed steps (the end-to-end legs overwrite them with
+    # the host pool's data)
+    sample = gpu_sample = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = OracleSample(w)
+        gpu_sample = sample.gpu_outputs(st)
+
     e2e = e2e_hidden = None
     if not args.no_e2e:
         pool = HostPool(st)
@@ -444,10 +452,6 @@ def run_ours(args, rank, world, local_rank):
                       f"{flush.numel() / 2**20:.0f} MiB buffer written between steps, outside "
                       "each step's events")}
     gen_per_step = (st.n_layers * (2 + (1 if w.sinks else 0))) if stream_qk else 0
-    sample = gpu_sample = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        sample = OracleSample(w)
-        gpu_sample = sample.gpu_outputs(st)
     del st
     if rank != 0:
         return None
