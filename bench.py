@@ -768,7 +768,6 @@ def time_graph(st, K: int, flush):
             "launches_per_step": lib_launches(st.w), "bit_equal_to_calls": same}
 
 
-
 def _time_calls(fn, sync, min_warm_s: float = 0.5, want_s: float = 1.5, min_iters: int = 3):
     """CUDA-event time of one fn() after at least min_warm_s (and two calls) of warm-up;
     the number of timed calls targets want_s.  Returns ms per call."""
