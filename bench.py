@@ -104,9 +104,16 @@ class ClockSampler:
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         lines = self.lines
+        widened = False
         if self.t0 is not None:
             # a line is read up to one sampling interval after the sample was taken
-            lines = [x for x in lines if self.t0 <= x[0] <= self.t1 + 0.05]
+            inside = [x for x in lines if self.t0 <= x[0] <= self.t1 + 0.05]
+            if not inside:
+                # a timed region shorter than the sampling interval: the samples taken
+                # within half a second of it
+                inside = [x for x in lines if self.t0 - 0.5 <= x[0] <= self.t1 + 0.5]
+                widened = True
+            lines = inside
         for _, ln in lines:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 9:
@@ -121,8 +128,11 @@ class ClockSampler:
                     reasons.add(n)
         if not sm:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        out = {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+               "samples": len(sm)}
+        if widened:
+            out["window"] = "timed region shorter than the 50 ms sampling: samples within 0.5 s of it"
+        return out
 
 
 # ------------------------------------------------------------------ workload

@@ -43,6 +43,22 @@ def test_parity_record_of_the_sample():
     assert abs(p["importance_max_rel_err"] - 0.05) < 1e-6
 
 
+def test_clock_summary_of_a_short_region():
+    # a timed region shorter than the sampling interval holds no sample: the summary
+    # takes the samples within half a second of it and says so
+    c = bench.ClockSampler(0)
+    c.lines = [(100.0, "0, 2070, 2070, 500.0, 0x0, Not Active, Not Active, Not Active, Not Active"),
+               (100.3, "0, 2060, 2070, 510.0, 0x0, Not Active, Not Active, Not Active, Active"),
+               (103.0, "0, 1000, 2070, 100.0, 0x0, Not Active, Not Active, Not Active, Not Active")]
+    c.window(100.1, 100.11)
+    out = c.summary()
+    assert out["samples"] == 2 and out["sm_mhz"] == 2065.0 and out["reasons"] == ["sw_power_cap"]
+    assert "window" in out
+    c.window(99.9, 100.35)
+    out = c.summary()
+    assert out["samples"] == 2 and "window" not in out
+
+
 def test_oracle_sample_long_prompt_uses_last_rows():
     # a 32768-token prompt exceeds the pair budget: one head per thread (8 here), its last
     # query rows only, the first row the one that keeps the pairs within budget

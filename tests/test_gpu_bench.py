@@ -38,6 +38,7 @@ def test_bench_line(args):
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"]["h2d_bytes_per_step"] > 0 and d["e2e"]["d2h_bytes_per_step"] > 0
     assert d["gpu_launches"] > 0
+    assert d["clocks"] and d["clocks"]["sm_mhz"] > 0 and "reasons" in d["clocks"]
     p = d["parity"]
     assert p["entropy_max_abs_err_nats"] <= p["tolerance"]["entropy_nats"]
     assert p["importance_max_rel_err"] <= p["tolerance"]["importance_rel"]
