@@ -22,7 +22,7 @@ def _lens(rng, B, hi):
     return [int(x) for x in lens]
 
 
-@pytest.mark.parametrize("seed", range(24))
+@pytest.mark.parametrize("seed", range(48))
 def test_sweep_importance(cuda_lib, seed):
     """Random (lengths, Hq / Hkv, d, head subset, self term, divisor), bf16 on the tensor
     cores, two layers accumulated."""
@@ -42,7 +42,7 @@ def test_sweep_importance(cuda_lib, seed):
     assert_importance(S, ref)
 
 
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(24))
 def test_sweep_entropy(cuda_lib, seed):
     """Random rows, vocabulary (not a multiple of anything) and row stride, bf16 and fp32."""
     rng = np.random.default_rng(2000 + seed)
@@ -62,7 +62,7 @@ def test_sweep_entropy(cuda_lib, seed):
     assert_entropy(H.cpu().numpy(), oracle.token_entropy(host, V=V))
 
 
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(24))
 def test_sweep_pool(cuda_lib, seed):
     """Random lengths (empty prompts included), hidden size and mix, bf16, with the head."""
     rng = np.random.default_rng(3000 + seed)
@@ -91,7 +91,7 @@ def test_sweep_pool(cuda_lib, seed):
     assert np.max(np.abs(pred.cpu().numpy() - y_ref)) <= 1.0
 
 
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(24))
 def test_sweep_lm_head(cuda_lib, seed):
     """Random rows, hidden size (a multiple of 64) and vocabulary for the entropy formed
     from hidden states."""
@@ -109,7 +109,7 @@ def test_sweep_lm_head(cuda_lib, seed):
     assert_entropy(H.cpu().numpy(), oracle.lm_head_entropy(bits(h), bits(W)))
 
 
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(24))
 def test_sweep_attn_forward(cuda_lib, seed):
     """Random lengths (empty prompts included), GQA ratio, self term, divisor, lse supplied
     or computed, one or two layers through the fused forward (bf16, d 128)."""
