@@ -37,8 +37,10 @@
 //   warp 19     adds the four lane quarters' column sums of every tile, in order, and
 //               writes the tile's partial slot
 // TMEM: S double-buffered (2 x 128 columns), O (128), P double-buffered (2 x 64 columns of
-// bf16 pairs): all 512.  Every mbarrier wait is bounded; on expiry the CTA records
-// ESTP_ERR_TIMEOUT and drains.
+// bf16 pairs): all 512.  Every mbarrier wait is bounded (a test may lower the limit of the
+// abortable waits through estp_set_wait_limit); on expiry the CTA records ESTP_ERR_TIMEOUT
+// and drains: the producer waits for the last copy into each Q, K and V slot, each issuer
+// for all its MMAs, before the TMEM is freed.
 #include <cstddef>
 
 #include "importance_tc.cuh"
